@@ -1,0 +1,242 @@
+/*
+ * dbw.h - C ABI of the GB300 (sm_103a) hot path of Dynamic Backup Workers.
+ *
+ * Method: C. Xu, G. Neglia, N. Sebastianelli, "Dynamic Backup Workers for
+ * Parallel Machine Learning" (arXiv 2004.14696).  One synchronous
+ * parameter-server (PS) iteration with n workers simulated on one GPU:
+ *
+ *   dbw_choose_b          Eqs. (13)-(19): b_t = n - k_t from the estimator state
+ *   dbw_worker_grads      Eq. (2): every worker's minibatch gradient -> G [n, ld]
+ *   dbw_select_fastest    Eq. (4): arrival order of the n gradients, the k kept
+ *   dbw_aggregate_update  Eqs. (3)-(4): masked mean + SGD step, fused with the
+ *                         partial sums of Eq. (10), ||g_t||^2 and ||g_j||^2
+ *   dbw_grad_stats        Eqs. (10)-(12) and Sect. 3.2: finishes the statistics
+ *                         and records them (and the order statistics) in the state
+ *
+ * Conventions shared by every call:
+ *  - Every pointer argument is a DEVICE pointer owned by the caller unless its
+ *    comment says "host".  The library never allocates in these calls; scratch
+ *    ("workspace", "partials") is caller memory sized by the *_bytes queries.
+ *  - Every compute call is asynchronous on ``stream`` (a cudaStream_t passed as
+ *    void*, NULL = legacy default stream) and returns an int status:
+ *      DBW_OK (0), DBW_EINVAL (bad argument, detected on the host before any
+ *      launch), DBW_EALIGN (a pointer or leading dimension violates the stated
+ *      alignment), DBW_ECUDA (a CUDA launch error), DBW_EUNSUPPORTED (device
+ *      is not sm_103).  dbw_last_error_string() describes the last failure of
+ *      the calling thread.  Nothing is launched when a call returns an error.
+ *  - Errors that can only be seen on the device (a device-resident b out of
+ *    range, a sample index out of range) never fault: they are clamped or
+ *    poisoned as documented per call and raise a bit in dbw_state.flags or
+ *    produce NaN in the outputs.
+ *  - Floating point: gradients, parameters and G are fp32 (GEMM operands
+ *    optionally bf16 with fp32 accumulation); estimator quantities are fp64.
+ */
+#ifndef DBW_H
+#define DBW_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DBW_OK 0
+#define DBW_EINVAL (-1)
+#define DBW_EALIGN (-2)
+#define DBW_ECUDA (-3)
+#define DBW_EUNSUPPORTED (-4)
+
+#define DBW_PREC_FP32 0 /* fp32 GEMM operands, fp32 accumulation */
+#define DBW_PREC_BF16 1 /* bf16 GEMM operands (RNE from fp32), fp32 accumulation */
+
+#define DBW_NMAX 1024 /* maximum number of workers n */
+#define DBW_DMAX 64   /* maximum window D of Eqs. (13)-(15) */
+#define DBW_LMAX 8    /* maximum number of layers */
+
+/* dbw_choose_b flags */
+#define DBW_CHOOSE_BLIND 1 /* B-DBW (Sect. 4): the gain of k is k itself */
+
+/* dbw_state.flags bits (sticky, OR-ed over iterations) */
+#define DBW_FLAG_K1 (1 << 0)        /* an iteration kept k = 1: Eq. (10) undefined, not recorded */
+#define DBW_FLAG_L_SKIPPED (1 << 1) /* an Eq. (12) value had denominator <= 0 or was not finite */
+#define DBW_FLAG_EMPTY_MASK (1 << 2) /* dbw_grad_stats saw no received worker: nothing recorded */
+#define DBW_FLAG_BAD_STATE (1 << 3)  /* state->n disagrees with the call's n (or is out of range) */
+
+/* indices into the stats_out vector of dbw_grad_stats (DBW_STATS_LEN doubles) */
+#define DBW_STAT_K 0       /* k_t, number of received gradients */
+#define DBW_STAT_SS 1      /* sum_l sum_{j<=k} ([g_j - g_t]_l)^2 (double sum of Eq. (10)) */
+#define DBW_STAT_GBAR_SQ 2 /* ||g_t||^2 */
+#define DBW_STAT_V 3       /* V^+ of Eq. (10) (NaN if k = 1) */
+#define DBW_STAT_N 4       /* ||grad F(w_t)||^2 ^+ of Eq. (11) (NaN if k = 1) */
+#define DBW_STAT_F 5       /* F^_t, mean minibatch loss of the received workers (Sect. 3.1) */
+#define DBW_STAT_L 6       /* L^+_t of Eq. (12) (NaN if not available / not recorded) */
+#define DBW_STAT_FLAGS 7   /* DBW_FLAG_* bits raised by this iteration */
+#define DBW_STAT_VCLOCK 8  /* virtual clock after this iteration: sum of T_(k_t) */
+#define DBW_STATS_LEN 9
+
+/*
+ * Estimator state carried by the PS from iteration to iteration (device memory,
+ * plain old data: save/restore by copying sizeof(dbw_state) bytes).
+ *
+ * Rings hold the most recently recorded "+" estimates of Eqs. (10), (11), (12);
+ * cnt* counts all values ever recorded, the newest sits at index (cnt-1) % DMAX.
+ * S[k-1] is the running sum of the k-th arrival time, c the number of observed
+ * time vectors, so that T^_k = S[k-1] / c (Eq. (17) under push-and-interrupt,
+ * where every k has c samples and the per-k means are already monotone).
+ */
+typedef struct dbw_state {
+    int32_t n;        /* workers */
+    int32_t D;        /* window of Eqs. (13)-(15), 1..DBW_DMAX */
+    int32_t t;        /* completed iterations */
+    int32_t k_last;   /* k_{t-1} */
+    int32_t c;        /* time vectors observed */
+    int32_t cntV, cntN, cntL;
+    int32_t flags;    /* sticky DBW_FLAG_* */
+    int32_t has_last; /* V_last / N_last hold iteration t-1's recorded estimates */
+    int32_t k_next;   /* k_t written by the last dbw_choose_b */
+    int32_t reserved;
+    double F_last;    /* F^_{t-1} */
+    double F_prev;    /* F^_{t-2} */
+    double N_last;    /* ||grad F||^2 ^+ of iteration t-1 */
+    double V_last;    /* V^+ of iteration t-1 */
+    double vclock;    /* virtual clock: sum over iterations of the k_t-th arrival time */
+    double ringV[DBW_DMAX];
+    double ringN[DBW_DMAX];
+    double ringL[DBW_DMAX];
+    double S[DBW_NMAX];
+} dbw_state;
+
+/* Text of the calling thread's last error ("" if none).  Host; never fails. */
+const char* dbw_last_error_string(void);
+
+/* ABI version (incremented on any signature or layout change). */
+int dbw_abi_version(void);
+
+/* ----------------------------------------------------------------------- model
+ * A fully connected ReLU network (Sect. 4 trains neural networks with the
+ * cross-entropy loss): widths[0] inputs, widths[1..L-1] hidden ReLU layers,
+ * widths[L] classes, L = num_layers in [1, DBW_LMAX].  Parameters are one flat
+ * fp32 vector w [d] in layer order, each layer W_l [out, in] row-major then
+ * b_l [out]; G rows use the same order.  widths is a HOST array.
+ */
+
+/* d for these widths, or -1 if an argument is invalid. */
+int64_t dbw_param_count(int num_layers, const int32_t* widths);
+
+/* Workspace bytes dbw_worker_grads needs for (widths, n, B, prec); 0 if invalid. */
+size_t dbw_worker_grads_workspace_bytes(int num_layers, const int32_t* widths, int n, int B, int prec);
+
+/*
+ * Eq. (2): g_{i,t} = (1/B) sum_{x in B_i} grad f(x, w_t) for every worker i.
+ *
+ *  w       [d] fp32 parameters w_t (16-byte aligned).
+ *  pool    [S, widths[0]] fp32 dataset features, row-major (16-byte aligned).
+ *  labels  [S] int32 class of each pool row.
+ *  idx     [n*B] int32 pool rows of the minibatches; worker i owns
+ *          idx[i*B .. i*B+B-1].  An index outside [0, S) or a label outside
+ *          [0, classes) makes that worker's loss and gradient NaN.
+ *  G       [n, ld] fp32 output, row i = g_{i,t}; ld >= d, ld % 4 == 0, 16-byte
+ *          aligned.  Columns d..ld-1 are not written.
+ *  loss    [n] fp32 output: each worker's minibatch mean loss (Sect. 3.1, F^_t).
+ *  ws      workspace of ws_bytes >= dbw_worker_grads_workspace_bytes(...),
+ *          256-byte aligned; contents are scratch.
+ *  prec    DBW_PREC_FP32 or DBW_PREC_BF16.
+ */
+int dbw_worker_grads(int num_layers, const int32_t* widths, int prec,
+                     const float* w, int64_t d,
+                     const float* pool, int64_t S, const int32_t* labels,
+                     const int32_t* idx, int n, int B,
+                     float* G, int64_t ld, float* loss,
+                     void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Eq. (4): the PS waits for the first k = n - b gradients.
+ * Arrival order is (times[i], i) ascending (ties go to the lower worker index).
+ *
+ *  times    [n] fp64 round-trip times of this iteration (finite, not NaN).
+ *  b        device int32 scalar, the number of backup workers; values outside
+ *           [0, n-1] are clamped into it.
+ *  order    [n] int32 out: order[r] = worker with arrival rank r.
+ *  mask     [n] uint8 out: 1 for the k received workers, else 0.
+ *  tsorted  [n] fp64 out: order statistics, tsorted[r] = times[order[r]];
+ *           tsorted[k-1] is the iteration's duration for every candidate k.
+ *  k_out    device int32 scalar out (nullable): the k actually used.
+ *  n in [1, DBW_NMAX].
+ */
+int dbw_select_fastest(const double* times, int n, const int32_t* b,
+                       int32_t* order, uint8_t* mask, double* tsorted,
+                       int32_t* k_out, void* stream);
+
+/* Bytes of the partials buffer dbw_aggregate_update needs on the current device. */
+size_t dbw_aggregate_partials_bytes(int n, int64_t d);
+
+/*
+ * Eqs. (3)-(4) fused with the statistics of Sect. 3.1, one pass over G:
+ *   g_t = (1/k) sum_{j: mask[j]} G[j, :]       (k = number of set mask bytes)
+ *   w   = w - lr * g_t                          (in place)
+ * and, into ``partials``, the per-block pieces of sum_j ||g_j||^2 (received
+ * rows), sum_l sum_j (G[j,l] - g_t[l])^2 and ||g_t||^2, which dbw_grad_stats
+ * reduces.  Column sums use a per-column shift (the first received row) so that
+ * the deviation sum does not cancel; cross-column sums are fp64.
+ *
+ *  G        [n, ld] fp32, ld % 4 == 0, 16-byte aligned; only received rows read.
+ *  mask     [n] uint8 from dbw_select_fastest (at least one byte set).
+ *  w        [d] fp32, updated in place (16-byte aligned).
+ *  gbar     [d] fp32 out (nullable, 16-byte aligned): g_t.
+ *  partials scratch of partials_bytes >= dbw_aggregate_partials_bytes(n, d),
+ *           256-byte aligned; consumed by the next dbw_grad_stats.
+ */
+int dbw_aggregate_update(const float* G, int64_t ld, int n, int64_t d,
+                         const uint8_t* mask, float lr, float* w, float* gbar,
+                         double* partials, size_t partials_bytes, void* stream);
+
+/* Initialise a device dbw_state for n workers and window D (k_0 = n). */
+int dbw_state_init(dbw_state* state, int n, int D, void* stream);
+
+/*
+ * End-of-iteration statistics (Sect. 3.1) and time bookkeeping (Sect. 3.2):
+ *   V^+ = SS / (k-1)                         Eq. (10)
+ *   ||grad F||^2^+ = max(||g_t||^2 - V^+/k, 0) Eq. (11)
+ *   F^_t = mean of loss[j] over received j    (summed in increasing j)
+ *   L^+_t from Eq. (12) with iteration t-1's estimates and F^_{t-1} - F^_t
+ * recorded into the state's rings (k = 1 and invalid Eq. (12) values are not
+ * recorded), S[r] += tsorted[r] for all r, c += 1, vclock += tsorted[k-1].
+ *
+ *  partials    the buffer the preceding dbw_aggregate_update of this iteration wrote.
+ *  mask, loss  [n] this iteration's selection and per-worker losses.
+ *  tsorted     [n] from dbw_select_fastest.
+ *  lr          the learning rate eta used by the update.
+ *  stats_out   [DBW_STATS_LEN] fp64 out (nullable), see DBW_STAT_*.
+ *  row_sqnorm  [n] fp64 out (nullable): ||g_j||^2 for received rows, NaN otherwise.
+ */
+int dbw_grad_stats(const double* partials, int n, const uint8_t* mask,
+                   const float* loss, const double* tsorted, double lr,
+                   dbw_state* state, double* stats_out, double* row_sqnorm,
+                   void* stream);
+
+/*
+ * Eqs. (16), (18), (19): choose k_t for the iteration about to start and write
+ * b_t = n - k_t to ``b_out`` (device int32 scalar) and to state->k_next.
+ *   G^_k  = (eta - q) N^ - q V^ / k,  q = L^ eta^2 / 2, with N^, V^, L^ the
+ *           window means of Eqs. (13)-(15) over the last min(D, recorded) values;
+ *   T^_k  = S[k-1] / c;
+ *   k_t   = argmax_{k: G^_k > 0} G^_k / T^_k (ties -> larger k), k_t = n if no
+ *           G^_k > 0 or any window is still empty (k_0 = k_1 = n);
+ *   Eq. (19): if t >= 2, F^_{t-1} > beta F^_{t-2} and k_{t-1} < n, then
+ *           k_t = max(k_t, k_{t-1} + 1).
+ * All fp64 operations are performed one at a time in this order (no fused
+ * multiply-add), so equal states give bit-identical b_t.
+ *
+ *  flags      0 or DBW_CHOOSE_BLIND (gain of k := k, Sect. 4's B-DBW).
+ *  ratio_out  [n] fp64 out (nullable): G^_k / T^_k for k = 1..n (NaN while a
+ *             window is empty).
+ */
+int dbw_choose_b(dbw_state* state, double lr, double beta, int flags,
+                 int32_t* b_out, double* ratio_out, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DBW_H */

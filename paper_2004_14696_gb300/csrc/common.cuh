@@ -1,0 +1,65 @@
+// Internal helpers shared by the CUDA translation units of libdbw.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "dbw.h"
+
+namespace dbw {
+
+// Records a message for dbw_last_error_string() and returns ``code``.
+int fail(int code, const char* fmt, ...);
+// Maps a pending launch error to DBW_ECUDA (with its text), else DBW_OK.
+int check_launch(const char* what);
+// Number of SMs of the current device (cached per device).
+int sm_count();
+// DBW_OK if the current device is sm_103 (compute capability 10.3), else DBW_EUNSUPPORTED.
+int check_device();
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline bool aligned256(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 255u) == 0; }
+inline cudaStream_t as_stream(void* s) { return reinterpret_cast<cudaStream_t>(s); }
+
+// ----------------------------------------------------------------- launchers
+// Selection (select.cu)
+cudaError_t launch_select(const double* times, int n, const int32_t* b, int32_t* order,
+                          uint8_t* mask, double* tsorted, int32_t* k_out, cudaStream_t st);
+
+// Aggregation (aggregate.cu)
+struct AggGeometry {
+    int blocks;           // persistent grid size
+    int rows_stride;      // n + 2: values per block in the partials
+    size_t bytes;         // total partials bytes
+};
+AggGeometry agg_geometry(int n, int64_t d);
+cudaError_t launch_aggregate(const float* G, int64_t ld, int n, int64_t d, const uint8_t* mask,
+                             float lr, float* w, float* gbar, double* partials,
+                             const AggGeometry& g, cudaStream_t st);
+
+// Estimator (estimator.cu)
+cudaError_t launch_state_init(dbw_state* s, int n, int D, cudaStream_t st);
+cudaError_t launch_grad_stats(const double* partials, int n, const uint8_t* mask, const float* loss,
+                              const double* tsorted, double lr, dbw_state* s, double* stats_out,
+                              double* row_sqnorm, cudaStream_t st);
+cudaError_t launch_choose_b(dbw_state* s, double lr, double beta, int flags, int32_t* b_out,
+                            double* ratio_out, cudaStream_t st);
+
+// Worker gradients (grads.cu)
+struct GradsPlan;
+size_t grads_workspace_bytes(int L, const int32_t* widths, int n, int B, int prec);
+int launch_worker_grads(int L, const int32_t* widths, int prec, const float* w, int64_t d,
+                        const float* pool, int64_t S, const int32_t* labels, const int32_t* idx,
+                        int n, int B, float* G, int64_t ld, float* loss, void* ws, size_t ws_bytes,
+                        cudaStream_t st);
+
+// Partials buffer layout shared by aggregate.cu and estimator.cu:
+//   int64 header[4] = {magic, blocks, n, reserved}
+//   double sums[n + 2]              reduced totals (written by dbw_grad_stats)
+//   double vals[(n + 2) * blocks]   per-block pieces, by quantity: vals[q * blocks + blk]
+//                                   q < n: ||g_q||^2, q = n: SS, q = n + 1: ||g_t||^2
+constexpr int64_t kPartialsMagic = 0x44425750415254LL;  // "DBWPART"
+constexpr int kPartialsHeader = 4;
+
+}  // namespace dbw

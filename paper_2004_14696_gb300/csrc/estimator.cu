@@ -1,0 +1,270 @@
+// The DBW estimator on the device (Sect. 3): end-of-iteration statistics
+// (Eqs. (10)-(12), time bookkeeping of Sect. 3.2) and the choice of k_t
+// (Eqs. (13)-(19)).  Everything is fp64 and runs in one CTA.
+//
+// This file is compiled with -fmad=false: every multiply and add below is a
+// separately rounded IEEE operation, performed in the order written, so that a
+// state reproduced elsewhere with the same operation order yields the same b_t
+// bit for bit.  The sequential pieces (window sums, the loss mean) run in one
+// thread on purpose: their summation order is part of that contract.
+#include <math.h>
+#include <math_constants.h>
+
+#include "common.cuh"
+
+namespace dbw {
+
+namespace {
+
+constexpr int kRedThreads = 256;
+
+__device__ __forceinline__ int ring_slot(int cnt_minus_v) { return cnt_minus_v % DBW_DMAX; }
+
+__device__ double window_mean(const double* ring, int cnt, int D) {
+    const int m = cnt < D ? cnt : D;
+    double acc = 0.0;
+    for (int v = 1; v <= m; ++v) acc = acc + ring[ring_slot(cnt - v)];
+    return acc / (double)m;
+}
+
+// Sum of the per-block pieces of one quantity, in a fixed order: thread t adds
+// blocks t, t + 256, ... sequentially, then a fixed pairwise tree.
+__global__ void __launch_bounds__(kRedThreads) reduce_partials_kernel(double* __restrict__ partials, int n) {
+    const int64_t* hdr = reinterpret_cast<const int64_t*>(partials);
+    double* sums = partials + kPartialsHeader;
+    if (hdr[0] != kPartialsMagic || hdr[2] != n || hdr[1] < 1 || hdr[1] > (1 << 20)) {
+        // not written by dbw_aggregate_update for this n: poison instead of reading
+        if (threadIdx.x == 0) sums[blockIdx.x] = CUDART_NAN;
+        return;
+    }
+    const int blocks = (int)hdr[1];
+    const double* vals = partials + kPartialsHeader + (n + 2) + (int64_t)blockIdx.x * blocks;
+    __shared__ double red[kRedThreads];
+    double s = 0.0;
+    for (int i = threadIdx.x; i < blocks; i += kRedThreads) s = s + vals[i];
+    red[threadIdx.x] = s;
+    __syncthreads();
+    for (int h = kRedThreads / 2; h > 0; h >>= 1) {
+        if (threadIdx.x < h) red[threadIdx.x] = red[threadIdx.x] + red[threadIdx.x + h];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) sums[blockIdx.x] = red[0];
+}
+
+__global__ void __launch_bounds__(1024) grad_stats_kernel(
+    const double* __restrict__ sums, int n, const uint8_t* __restrict__ mask,
+    const float* __restrict__ loss, const double* __restrict__ tsorted, double lr,
+    dbw_state* __restrict__ st, double* __restrict__ stats_out, double* __restrict__ row_sqnorm) {
+    __shared__ int k_s;
+    const int tid = threadIdx.x;
+    if (tid == 0) {
+        int k = 0;
+        for (int j = 0; j < n; ++j) k += mask[j] ? 1 : 0;
+        k_s = k;
+        if (k == 0 || st->n != n) {
+            st->flags |= (k == 0 ? DBW_FLAG_EMPTY_MASK : 0) | (st->n != n ? DBW_FLAG_BAD_STATE : 0);
+            k_s = 0;
+        }
+    }
+    __syncthreads();
+    if (k_s == 0) return;
+    if (tid == 0) {
+        const int k = k_s;
+        double acc = 0.0;
+        for (int j = 0; j < n; ++j)
+            if (mask[j]) acc = acc + (double)loss[j];
+        const double SS = sums[n];
+        const double g2 = sums[n + 1];
+        const double F = acc / (double)k;
+        double V = CUDART_NAN, N = CUDART_NAN, L = CUDART_NAN;
+        int flags = 0;
+        if (k >= 2) {
+            V = SS / (double)(k - 1);                         // Eq. (10)
+            const double x = g2 - V / (double)k;              // Eq. (11)
+            N = x > 0.0 ? x : 0.0;
+        } else {
+            flags |= DBW_FLAG_K1;
+        }
+        if (st->t >= 1 && st->has_last) {                     // Eq. (12)
+            const double num = 2.0 * ((lr * st->N_last) - (st->F_last - F));
+            const double den = (lr * lr) * (st->N_last + (st->V_last / (double)st->k_last));
+            if (den > 0.0) L = num / den;
+            if (!(den > 0.0 && isfinite(L))) {
+                L = CUDART_NAN;
+                flags |= DBW_FLAG_L_SKIPPED;
+            } else {
+                st->ringL[st->cntL % DBW_DMAX] = L;
+                st->cntL += 1;
+            }
+        }
+        if (k >= 2) {
+            st->ringV[st->cntV % DBW_DMAX] = V;
+            st->cntV += 1;
+            st->ringN[st->cntN % DBW_DMAX] = N;
+            st->cntN += 1;
+            st->N_last = N;
+            st->V_last = V;
+            st->has_last = 1;
+        } else {
+            st->N_last = CUDART_NAN;
+            st->V_last = CUDART_NAN;
+            st->has_last = 0;
+        }
+        st->c += 1;
+        st->vclock = st->vclock + tsorted[k - 1];
+        st->F_prev = st->F_last;
+        st->F_last = F;
+        st->k_last = k;
+        st->t += 1;
+        st->flags |= flags;
+        if (stats_out) {
+            stats_out[DBW_STAT_K] = (double)k;
+            stats_out[DBW_STAT_SS] = SS;
+            stats_out[DBW_STAT_GBAR_SQ] = g2;
+            stats_out[DBW_STAT_V] = V;
+            stats_out[DBW_STAT_N] = N;
+            stats_out[DBW_STAT_F] = F;
+            stats_out[DBW_STAT_L] = L;
+            stats_out[DBW_STAT_FLAGS] = (double)flags;
+            stats_out[DBW_STAT_VCLOCK] = st->vclock;
+        }
+    }
+    // Sect. 3.2: every arrival is observed, S[r] accumulates the r-th order statistic
+    for (int r = tid; r < n; r += blockDim.x) st->S[r] = st->S[r] + tsorted[r];
+    if (row_sqnorm)
+        for (int j = tid; j < n; j += blockDim.x) row_sqnorm[j] = mask[j] ? sums[j] : CUDART_NAN;
+}
+
+__global__ void __launch_bounds__(1024) choose_b_kernel(dbw_state* __restrict__ st, double lr, double beta,
+                                                        int flags, int32_t* __restrict__ b_out,
+                                                        double* __restrict__ ratio_out) {
+    __shared__ double Vh_s, Nh_s, q_s;
+    __shared__ int ready_s;
+    __shared__ double best_r[32];
+    __shared__ int best_k[32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int n = st->n;
+    if (n < 1 || n > DBW_NMAX || st->D < 1 || st->D > DBW_DMAX || st->cntV < 0 || st->cntN < 0 ||
+        st->cntL < 0 || st->c < 0) {
+        if (tid == 0) st->flags |= DBW_FLAG_BAD_STATE;
+        return;
+    }
+    const bool blind = (flags & DBW_CHOOSE_BLIND) != 0;
+    if (tid == 0) {
+        int ready;
+        if (blind) {
+            ready = st->c > 0;
+        } else {
+            ready = st->cntV > 0 && st->cntN > 0 && st->cntL > 0 && st->c > 0;
+            if (ready) {
+                Vh_s = window_mean(st->ringV, st->cntV, st->D);   // Eq. (13)
+                Nh_s = window_mean(st->ringN, st->cntN, st->D);   // Eq. (14)
+                const double Lh = window_mean(st->ringL, st->cntL, st->D);   // Eq. (15)
+                q_s = ((Lh * lr) * lr) / 2.0;
+            }
+        }
+        ready_s = ready;
+    }
+    __syncthreads();
+    const int ready = ready_s;
+    const double c = (double)st->c;
+    // candidate of this thread: k = tid + 1
+    double my_r = -CUDART_INF;
+    int my_k = 0;   // 0 = not eligible
+    for (int k = tid + 1; k <= n; k += blockDim.x) {
+        double ratio = CUDART_NAN;
+        bool elig = false;
+        if (ready) {
+            const double T = st->S[k - 1] / c;                    // T^_k
+            if (blind) {
+                ratio = (double)k / T;
+                elig = true;
+            } else {
+                const double gain = ((lr - q_s) * Nh_s) - (q_s * (Vh_s / (double)k));   // Eq. (16)
+                ratio = gain / T;
+                elig = gain > 0.0;
+            }
+        }
+        if (ratio_out) ratio_out[k - 1] = ratio;
+        if (elig && (my_k == 0 || ratio > my_r || (ratio == my_r && k > my_k))) {
+            my_r = ratio;
+            my_k = k;
+        }
+    }
+    // Eq. (18): lexicographic max of (eligible, ratio, k) across the CTA
+    for (int o = 16; o > 0; o >>= 1) {
+        const double r2 = __shfl_xor_sync(0xffffffffu, my_r, o);
+        const int k2 = __shfl_xor_sync(0xffffffffu, my_k, o);
+        if (k2 != 0 && (my_k == 0 || r2 > my_r || (r2 == my_r && k2 > my_k))) {
+            my_r = r2;
+            my_k = k2;
+        }
+    }
+    if (lane == 0) {
+        best_r[warp] = my_r;
+        best_k[warp] = my_k;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        int kstar = 0;
+        double rbest = -CUDART_INF;
+        for (int wv = 0; wv < (int)(blockDim.x >> 5); ++wv) {
+            const int k2 = best_k[wv];
+            const double r2 = best_r[wv];
+            if (k2 != 0 && (kstar == 0 || r2 > rbest || (r2 == rbest && k2 > kstar))) {
+                rbest = r2;
+                kstar = k2;
+            }
+        }
+        if (kstar == 0) kstar = n;                                // R3 / R7: k = n
+        if (st->t >= 2 && st->F_last > beta * st->F_prev && st->k_last < n) {   // Eq. (19)
+            const int kg = st->k_last + 1;
+            if (kg > kstar) kstar = kg;
+        }
+        if (kstar > n) kstar = n;
+        st->k_next = kstar;
+        *b_out = n - kstar;
+    }
+}
+
+__global__ void state_init_kernel(dbw_state* st, int n, int D) {
+    double* raw = reinterpret_cast<double*>(st);
+    const int nwords = (int)(sizeof(dbw_state) / sizeof(double));
+    for (int i = threadIdx.x; i < nwords; i += blockDim.x) raw[i] = 0.0;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        st->n = n;
+        st->D = D;
+        st->k_next = n;
+        st->F_last = CUDART_NAN;
+        st->F_prev = CUDART_NAN;
+        st->N_last = CUDART_NAN;
+        st->V_last = CUDART_NAN;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_state_init(dbw_state* s, int n, int D, cudaStream_t st) {
+    state_init_kernel<<<1, 256, 0, st>>>(s, n, D);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_grad_stats(const double* partials, int n, const uint8_t* mask, const float* loss,
+                              const double* tsorted, double lr, dbw_state* s, double* stats_out,
+                              double* row_sqnorm, cudaStream_t st) {
+    double* sums = const_cast<double*>(partials) + kPartialsHeader;
+    reduce_partials_kernel<<<n + 2, kRedThreads, 0, st>>>(sums - kPartialsHeader, n);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    grad_stats_kernel<<<1, 1024, 0, st>>>(sums, n, mask, loss, tsorted, lr, s, stats_out, row_sqnorm);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_choose_b(dbw_state* s, double lr, double beta, int flags, int32_t* b_out,
+                            double* ratio_out, cudaStream_t st) {
+    choose_b_kernel<<<1, 1024, 0, st>>>(s, lr, beta, flags, b_out, ratio_out);
+    return cudaGetLastError();
+}
+
+}  // namespace dbw

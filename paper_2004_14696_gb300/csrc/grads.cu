@@ -1,0 +1,388 @@
+// Eq. (2) for all n workers at once: g_i = (1/B) sum_{x in B_i} grad f(x, w).
+//
+// The n workers share w, so their minibatches are stacked into one batch of
+// M = n * B rows and every forward and input-gradient GEMM is a single GEMM over
+// M rows.  Only the weight gradient is per worker: G[i, W_l] = dZ_l[i]^T A_{l-1}[i]
+// with K = B, a batched GEMM over the n workers that writes G directly.
+//
+//   gather     X = pool[idx]                                (fp32 or bf16)
+//   forward    Z_l = A_{l-1} W_l^T + b_l, A_l = ReLU(Z_l)   (last layer: fp32 logits)
+//   loss       per-sample cross entropy, loss_i = mean over worker i's B samples,
+//              dZ_L = (softmax - onehot) / B
+//   backward   G[i, W_l] = dZ_l[i]^T A_{l-1}[i],  G[i, b_l] = sum_rows dZ_l[i],
+//              dZ_{l-1} = (dZ_l W_l) * 1[A_{l-1} > 0]      (ReLU'(0) = 0)
+//
+// GEMMs here are the SIMT path (fp32 FFMA on fp32 or bf16 operands); the bf16
+// configurations can instead run the tcgen05 kernels of gemm_tc.cu.
+#include <math.h>
+
+#include "common.cuh"
+#include "grads.cuh"
+
+namespace dbw {
+
+namespace {
+
+template <typename T> __device__ __forceinline__ float to_f(T v);
+template <> __device__ __forceinline__ float to_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
+template <typename T> __device__ __forceinline__ T from_f(float v);
+template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+
+// ------------------------------------------------------------------ gather
+// X[m, :] = pool[idx[m], :].  An index outside [0, S) reads row 0; the loss
+// kernel poisons that worker.
+template <typename T>
+__global__ void gather_kernel(const float* __restrict__ pool, int64_t S, int in, const int32_t* __restrict__ idx,
+                              int M, T* __restrict__ X) {
+    for (int m = blockIdx.y; m < M; m += gridDim.y) {
+        int64_t r = idx[m];
+        if (r < 0 || r >= S) r = 0;
+        const float* src = pool + r * in;
+        T* dst = X + (int64_t)m * in;
+        for (int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4; c < in; c += gridDim.x * blockDim.x * 4) {
+            if (c + 3 < in) {
+                const float4 v = *reinterpret_cast<const float4*>(src + c);
+                dst[c] = from_f<T>(v.x);
+                dst[c + 1] = from_f<T>(v.y);
+                dst[c + 2] = from_f<T>(v.z);
+                dst[c + 3] = from_f<T>(v.w);
+            } else {
+                for (int e = c; e < in; ++e) dst[e] = from_f<T>(src[e]);
+            }
+        }
+    }
+}
+
+// bf16 copy of the weight matrices (same flat layout as w; bias slots unused).
+__global__ void cast_bf16_kernel(const float* __restrict__ w, int64_t d, __nv_bfloat16* __restrict__ wb) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < d; i += (int64_t)gridDim.x * blockDim.x)
+        wb[i] = __float2bfloat16_rn(w[i]);
+}
+
+// ------------------------------------------------------------------ SIMT GEMM
+// C[m, n] = sum_k A(m, k) B(k, n) over a 128 x 128 tile per CTA, 16-deep K
+// slices staged in shared memory as fp32, 8 x 8 outputs per thread.
+//   A_K: A(m,k) = A[m*lda + k]   else A(m,k) = A[k*lda + m]
+//   B_K: B(k,n) = B[n*ldb + k]   else B(k,n) = B[k*ldb + n]
+// blockIdx.z is a batch index (offsets batchA / batchB).
+constexpr int BM = 128, BN = 128, BK = 16;
+
+template <typename T, bool A_K, bool B_K, class Epi>
+__global__ void __launch_bounds__(256) gemm_simt_kernel(int M, int N, int K, const T* __restrict__ A, int64_t lda,
+                                                        int64_t batchA, const T* __restrict__ B, int64_t ldb,
+                                                        int64_t batchB, Epi epi) {
+    __shared__ __align__(16) float As[BK][BM];
+    __shared__ __align__(16) float Bs[BK][BN];
+    const int z = blockIdx.z;
+    A += (int64_t)z * batchA;
+    B += (int64_t)z * batchB;
+    const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
+    const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+    float acc[8][8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+
+    for (int k0 = 0; k0 < K; k0 += BK) {
+#pragma unroll
+        for (int e = tid; e < BM * BK; e += 256) {
+            int mm, kk;
+            if (A_K) { mm = e / BK; kk = e % BK; } else { kk = e / BM; mm = e % BM; }
+            const int gm = m0 + mm, gk = k0 + kk;
+            float v = 0.f;
+            if (gm < M && gk < K) v = to_f<T>(A_K ? A[(int64_t)gm * lda + gk] : A[(int64_t)gk * lda + gm]);
+            As[kk][mm] = v;
+        }
+#pragma unroll
+        for (int e = tid; e < BN * BK; e += 256) {
+            int nn, kk;
+            if (B_K) { nn = e / BK; kk = e % BK; } else { kk = e / BN; nn = e % BN; }
+            const int gn = n0 + nn, gk = k0 + kk;
+            float v = 0.f;
+            if (gn < N && gk < K) v = to_f<T>(B_K ? B[(int64_t)gn * ldb + gk] : B[(int64_t)gk * ldb + gn]);
+            Bs[kk][nn] = v;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int kk = 0; kk < BK; ++kk) {
+            const float4 a0 = *reinterpret_cast<const float4*>(&As[kk][ty * 4]);
+            const float4 a1 = *reinterpret_cast<const float4*>(&As[kk][64 + ty * 4]);
+            const float4 b0 = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
+            const float4 b1 = *reinterpret_cast<const float4*>(&Bs[kk][64 + tx * 4]);
+            const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+            const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const int gm = m0 + (i < 4 ? ty * 4 + i : 64 + ty * 4 + (i - 4));
+        if (gm >= M) continue;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const int gn = n0 + (j < 4 ? tx * 4 + j : 64 + tx * 4 + (j - 4));
+            if (gn < N) epi(z, gm, gn, acc[i][j]);
+        }
+    }
+}
+
+// forward hidden layer: A_l = ReLU(C + b)
+template <typename T>
+struct EpiHidden {
+    const float* bias;
+    T* out;
+    int ldo;
+    __device__ __forceinline__ void operator()(int, int m, int n, float v) const {
+        v += bias[n];
+        out[(int64_t)m * ldo + n] = from_f<T>(v > 0.f ? v : 0.f);
+    }
+};
+// forward last layer: logits = C + b (fp32)
+struct EpiLogits {
+    const float* bias;
+    float* out;
+    int ldo;
+    __device__ __forceinline__ void operator()(int, int m, int n, float v) const {
+        out[(int64_t)m * ldo + n] = v + bias[n];
+    }
+};
+// input gradient: dZ_{l-1} = C * 1[A_{l-1} > 0]  (a product, so a NaN-poisoned row stays NaN)
+template <typename T>
+struct EpiDx {
+    const T* act;
+    T* out;
+    int ldo;
+    __device__ __forceinline__ void operator()(int, int m, int n, float v) const {
+        const float a = to_f<T>(act[(int64_t)m * ldo + n]);
+        out[(int64_t)m * ldo + n] = from_f<T>(v * (a > 0.f ? 1.f : 0.f));
+    }
+};
+// weight gradient of worker z: G[z, off + o * in + c]
+struct EpiDW {
+    float* G;
+    int64_t ldG;
+    int64_t off;
+    int in;
+    __device__ __forceinline__ void operator()(int z, int o, int c, float v) const {
+        G[(int64_t)z * ldG + off + (int64_t)o * in + c] = v;
+    }
+};
+
+// ------------------------------------------------------------------ loss
+// One CTA per worker.  Per sample: stable log-softmax cross entropy, and
+// dZ = (softmax - onehot) / B.  The worker's loss is the mean of its B sample
+// losses, summed in sample order.  A sample index outside [0, S) or a label
+// outside [0, C) makes the worker's loss and dZ rows NaN.
+template <typename T>
+__global__ void __launch_bounds__(256) softmax_xent_kernel(const float* __restrict__ logits, int C, int B,
+                                                           const int32_t* __restrict__ idx, int64_t S,
+                                                           const int32_t* __restrict__ labels,
+                                                           float* __restrict__ sample_loss, T* __restrict__ dZ,
+                                                           float* __restrict__ loss) {
+    const int i = blockIdx.x;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    __shared__ int bad_s;
+    if (threadIdx.x == 0) bad_s = 0;
+    __syncthreads();
+    const float invB = 1.0f / (float)B;
+    for (int r = warp; r < B; r += nw) {
+        const int64_t row = (int64_t)i * B + r;
+        const int64_t sidx = idx[row];
+        int y = -1;
+        if (sidx >= 0 && sidx < S) y = labels[sidx];
+        const bool bad = (y < 0 || y >= C);
+        const float* z = logits + row * C;
+        float mx = -INFINITY;
+        for (int c = lane; c < C; c += 32) mx = fmaxf(mx, z[c]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        float se = 0.f;
+        for (int c = lane; c < C; c += 32) se += expf(z[c] - mx);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
+        const float inv_se = 1.0f / se;
+        for (int c = lane; c < C; c += 32) {
+            float g = expf(z[c] - mx) * inv_se;
+            if (c == y) g -= 1.0f;
+            dZ[row * C + c] = from_f<T>(bad ? NAN : g * invB);
+        }
+        if (lane == 0) {
+            sample_loss[row] = bad ? NAN : (mx + logf(se)) - z[y];
+            if (bad) bad_s = 1;
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float acc = 0.f;
+        for (int r = 0; r < B; ++r) acc += sample_loss[(int64_t)i * B + r];
+        loss[i] = bad_s ? NAN : acc * invB;
+    }
+}
+
+// ------------------------------------------------------------------ bias gradient
+// G[i, offb + o] = sum_{r < B} dZ[i*B + r, o], summed in row order.
+template <typename T>
+__global__ void bias_grad_kernel(const T* __restrict__ dZ, int out, int B, float* __restrict__ G, int64_t ldG,
+                                 int64_t offb) {
+    const int i = blockIdx.y;
+    const int o = blockIdx.x * blockDim.x + threadIdx.x;
+    if (o >= out) return;
+    const T* p = dZ + (int64_t)i * B * out + o;
+    float acc = 0.f;
+    for (int r = 0; r < B; ++r) acc += to_f<T>(p[(int64_t)r * out]);
+    G[(int64_t)i * ldG + offb + o] = acc;
+}
+
+template <typename T, bool A_K, bool B_K, class Epi>
+cudaError_t run_gemm(int M, int N, int K, const T* A, int64_t lda, int64_t batchA, const T* B, int64_t ldb,
+                     int64_t batchB, int batch, Epi epi, cudaStream_t st) {
+    dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM, batch);
+    gemm_simt_kernel<T, A_K, B_K, Epi><<<grid, 256, 0, st>>>(M, N, K, A, lda, batchA, B, ldb, batchB, epi);
+    return cudaGetLastError();
+}
+
+template <typename T>
+int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int64_t S, const int32_t* labels,
+                      const int32_t* idx, float* G, int64_t ld, float* loss, char* ws, cudaStream_t st) {
+    const int L = P.L;
+    const int M = P.M;
+    const int B = P.B;
+    T* X = reinterpret_cast<T*>(ws + P.off_x);
+    float* logits = reinterpret_cast<float*>(ws + P.off_logits);
+    float* sloss = reinterpret_cast<float*>(ws + P.off_sloss);
+    T* dz[2] = {reinterpret_cast<T*>(ws + P.off_dz[0]), reinterpret_cast<T*>(ws + P.off_dz[1])};
+    const T* wop;
+    if (sizeof(T) == 2) {
+        __nv_bfloat16* wb = reinterpret_cast<__nv_bfloat16*>(ws + P.off_wb);
+        cast_bf16_kernel<<<4 * sm_count(), 256, 0, st>>>(w, P.d, wb);
+        wop = reinterpret_cast<const T*>(wb);
+    } else {
+        wop = reinterpret_cast<const T*>(w);
+    }
+    {
+        const int in = P.widths[0];
+        dim3 grid((in + 1023) / 1024, M < 65535 ? M : 65535);
+        gather_kernel<T><<<grid, 256, 0, st>>>(pool, S, in, idx, M, X);
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "gather launch: %s", cudaGetErrorString(e));
+
+    // forward
+    const T* Ain = X;
+    for (int l = 0; l < L; ++l) {
+        const int fin = P.widths[l], fout = P.widths[l + 1];
+        const T* W = wop + P.offW[l];
+        const float* bias = w + P.offb[l];
+        if (l < L - 1) {
+            T* Aout = reinterpret_cast<T*>(ws + P.off_act[l + 1]);
+            e = run_gemm<T, true, true>(M, fout, fin, Ain, fin, 0, W, fin, 0, 1, EpiHidden<T>{bias, Aout, fout}, st);
+            Ain = Aout;
+        } else {
+            e = run_gemm<T, true, true>(M, fout, fin, Ain, fin, 0, W, fin, 0, 1, EpiLogits{bias, logits, fout}, st);
+        }
+        if (e != cudaSuccess) return fail(DBW_ECUDA, "forward GEMM %d: %s", l, cudaGetErrorString(e));
+    }
+    const int C = P.widths[L];
+    softmax_xent_kernel<T><<<P.n, 256, 0, st>>>(logits, C, B, idx, S, labels, sloss, dz[0], loss);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "loss launch: %s", cudaGetErrorString(e));
+
+    // backward
+    int cur = 0;
+    for (int l = L - 1; l >= 0; --l) {
+        const int fin = P.widths[l], fout = P.widths[l + 1];
+        const T* Aprev = (l == 0) ? X : reinterpret_cast<const T*>(ws + P.off_act[l]);
+        const T* dZl = dz[cur];
+        // per-worker weight gradient: M' = fout, N' = fin, K = B; A(o, r) = dZ[r*fout + o], B(r, c) = A[r*fin + c]
+        e = run_gemm<T, false, false>(fout, fin, B, dZl, fout, (int64_t)B * fout, Aprev, fin, (int64_t)B * fin,
+                                      P.n, EpiDW{G, ld, P.offW[l], fin}, st);
+        if (e != cudaSuccess) return fail(DBW_ECUDA, "dW GEMM %d: %s", l, cudaGetErrorString(e));
+        bias_grad_kernel<T><<<dim3((fout + 127) / 128, P.n), 128, 0, st>>>(dZl, fout, B, G, ld, P.offb[l]);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return fail(DBW_ECUDA, "bias grad %d: %s", l, cudaGetErrorString(e));
+        if (l > 0) {
+            // dZ_{l-1}[m, c] = sum_o dZ_l[m, o] W_l[o, c]: A(m, o) = dZ[m*fout + o], B(o, c) = W[o*fin + c]
+            T* dnext = dz[cur ^ 1];
+            e = run_gemm<T, true, false>(M, fin, fout, dZl, fout, 0, wop + P.offW[l], fin, 0, 1,
+                                         EpiDx<T>{Aprev, dnext, fin}, st);
+            if (e != cudaSuccess) return fail(DBW_ECUDA, "dX GEMM %d: %s", l, cudaGetErrorString(e));
+            cur ^= 1;
+        }
+    }
+    return DBW_OK;
+}
+
+}  // namespace
+
+bool make_grads_plan(int L, const int32_t* widths, int n, int B, int prec, GradsPlan* P) {
+    if (L < 1 || L > DBW_LMAX || n < 1 || n > DBW_NMAX || B < 1) return false;
+    if (prec != DBW_PREC_FP32 && prec != DBW_PREC_BF16) return false;
+    P->L = L;
+    P->n = n;
+    P->B = B;
+    P->prec = prec;
+    const int64_t M = (int64_t)n * B;
+    if (M > (1LL << 30)) return false;
+    P->M = (int)M;
+    int maxw = 0;
+    int64_t off = 0;
+    for (int l = 0; l <= L; ++l) {
+        if (widths[l] < 1 || widths[l] > (1 << 20)) return false;
+        P->widths[l] = widths[l];
+        if (widths[l] > maxw) maxw = widths[l];
+    }
+    if (widths[L] < 2) return false;
+    for (int l = 0; l < L; ++l) {
+        P->offW[l] = off;
+        off += (int64_t)widths[l + 1] * widths[l];
+        P->offb[l] = off;
+        off += widths[l + 1];
+    }
+    P->d = off;
+    const size_t es = prec == DBW_PREC_BF16 ? 2 : 4;
+    size_t cur = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = cur;
+        cur += (bytes + 255) / 256 * 256;
+        return at;
+    };
+    P->off_x = take((size_t)M * widths[0] * es);
+    P->off_act[0] = P->off_x;
+    for (int l = 1; l < L; ++l) P->off_act[l] = take((size_t)M * widths[l] * es);
+    P->off_logits = take((size_t)M * widths[L] * 4);
+    P->off_sloss = take((size_t)M * 4);
+    P->off_dz[0] = take((size_t)M * maxw * es);
+    P->off_dz[1] = take((size_t)M * maxw * es);
+    P->off_wb = prec == DBW_PREC_BF16 ? take((size_t)P->d * 2) : 0;
+    P->ws_bytes = cur;
+    return true;
+}
+
+size_t grads_workspace_bytes(int L, const int32_t* widths, int n, int B, int prec) {
+    GradsPlan P;
+    if (!make_grads_plan(L, widths, n, B, prec, &P)) return 0;
+    return P.ws_bytes;
+}
+
+int launch_worker_grads(int L, const int32_t* widths, int prec, const float* w, int64_t d, const float* pool,
+                        int64_t S, const int32_t* labels, const int32_t* idx, int n, int B, float* G, int64_t ld,
+                        float* loss, void* ws, size_t ws_bytes, cudaStream_t st) {
+    GradsPlan P;
+    if (!make_grads_plan(L, widths, n, B, prec, &P)) return fail(DBW_EINVAL, "dbw_worker_grads: invalid model shape");
+    if (P.d != d) return fail(DBW_EINVAL, "dbw_worker_grads: d = %lld but the widths give %lld", (long long)d,
+                              (long long)P.d);
+    if (ws_bytes < P.ws_bytes)
+        return fail(DBW_EINVAL, "dbw_worker_grads: workspace %zu bytes < %zu needed", ws_bytes, P.ws_bytes);
+    if (prec == DBW_PREC_BF16)
+        return worker_grads_impl<__nv_bfloat16>(P, w, pool, S, labels, idx, G, ld, loss, static_cast<char*>(ws), st);
+    return worker_grads_impl<float>(P, w, pool, S, labels, idx, G, ld, loss, static_cast<char*>(ws), st);
+}
+
+}  // namespace dbw

@@ -1,0 +1,104 @@
+"""One DBW parameter-server iteration as a sequence of libdbw calls.
+
+``Iteration`` owns the device buffers of one workload (G, w, workspace,
+partials, estimator state) and issues, per step, the five C-ABI calls in the
+paper's order (Sect. 3: b_t is chosen right after w_t is available):
+
+    dbw_choose_b -> dbw_worker_grads -> dbw_select_fastest
+                 -> dbw_aggregate_update -> dbw_grad_stats
+
+Python only sequences the calls and owns memory through torch; every step of
+the computation runs in libdbw's kernels on the current CUDA stream.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import dbw, inputs
+from .workloads import Workload
+
+
+class Iteration:
+    def __init__(self, wl: Workload, device="cuda", static_b=None, blind=False, keep_gbar=False,
+                 pool=None, labels=None, w0=None):
+        self.wl = wl
+        self.device = torch.device(device)
+        n, d, ld = wl.n, wl.d, wl.ld
+        self.n, self.d, self.ld = n, d, ld
+        self.static_b = static_b
+        self.blind = blind
+        if pool is None:
+            pool = inputs.feature_pool(wl.seed, wl.S, wl.widths[0], wl.feature_dist)
+        if labels is None:
+            labels = inputs.label_pool(wl.seed, wl.S, wl.classes)
+        if w0 is None:
+            w0 = inputs.kaiming_uniform_params(wl.seed, wl.widths)
+        self.pool = torch.as_tensor(pool).to(self.device)
+        self.labels = torch.as_tensor(labels).to(self.device)
+        self.w = torch.as_tensor(w0).to(self.device).clone()
+        self.G = torch.empty((n, ld), dtype=torch.float32, device=self.device)
+        self.loss = torch.empty(n, dtype=torch.float32, device=self.device)
+        self.ws = torch.empty(dbw.dbw_worker_grads_workspace_bytes(wl.widths, n, wl.B, wl.prec),
+                              dtype=torch.uint8, device=self.device)
+        self.partials = torch.empty(dbw.dbw_aggregate_partials_bytes(n, d), dtype=torch.uint8, device=self.device)
+        self.state = dbw.new_state(n, wl.D, self.device)
+        self.b = torch.zeros(1, dtype=torch.int32, device=self.device)
+        if static_b is not None:
+            self.b.fill_(int(static_b))
+        self.k = torch.zeros(1, dtype=torch.int32, device=self.device)
+        self.order = torch.empty(n, dtype=torch.int32, device=self.device)
+        self.mask = torch.empty(n, dtype=torch.uint8, device=self.device)
+        self.tsorted = torch.empty(n, dtype=torch.float64, device=self.device)
+        self.ratio = torch.empty(n, dtype=torch.float64, device=self.device)
+        self.stats = torch.empty(dbw.STATS_LEN, dtype=torch.float64, device=self.device)
+        self.row_sqnorm = torch.empty(n, dtype=torch.float64, device=self.device)
+        self.gbar = torch.empty(d, dtype=torch.float32, device=self.device) if keep_gbar else None
+        # per-step inputs (device copies written by the caller or by load_inputs)
+        self.idx = torch.empty(n * wl.B, dtype=torch.int32, device=self.device)
+        self.times = torch.empty(n, dtype=torch.float64, device=self.device)
+
+    # ------------------------------------------------------------ inputs
+    def host_inputs(self, t):
+        wl = self.wl
+        idx = inputs.minibatch_indices(wl.seed, t, wl.n, wl.B, wl.S)
+        times = inputs.completion_times(wl.seed, t, wl.n, wl.time_model, **wl.time_params)
+        return idx, times
+
+    def load_inputs(self, t):
+        idx, times = self.host_inputs(t)
+        self.idx.copy_(torch.from_numpy(idx))
+        self.times.copy_(torch.from_numpy(times))
+
+    # ------------------------------------------------------------ one iteration
+    def step(self, idx=None, times=None, stream=None):
+        """Issue one iteration; idx / times default to the buffers self.idx / self.times."""
+        wl = self.wl
+        idx = self.idx if idx is None else idx
+        times = self.times if times is None else times
+        if self.static_b is None:
+            dbw.dbw_choose_b(self.state, wl.lr, wl.beta, self.b, self.ratio,
+                             dbw.CHOOSE_BLIND if self.blind else 0, stream)
+        dbw.dbw_worker_grads(wl.widths, wl.prec, self.w, self.pool, self.labels, idx, wl.n, wl.B, self.G,
+                             self.loss, self.ws, stream)
+        dbw.dbw_select_fastest(times, self.b, self.order, self.mask, self.tsorted, self.k, stream)
+        dbw.dbw_aggregate_update(self.G, wl.n, self.d, self.mask, wl.lr, self.w, self.partials, self.gbar, stream)
+        dbw.dbw_grad_stats(self.partials, wl.n, self.mask, self.loss, self.tsorted, wl.lr, self.state, self.stats,
+                           self.row_sqnorm, stream)
+
+    def launches_per_step(self):
+        """Kernels libdbw launches per step (for the bench's launch count)."""
+        L = len(self.wl.widths) - 1
+        grads = 1 + L + 1 + L + L + (L - 1)          # gather, fwd, loss, dW, bias, dX
+        if self.wl.prec == dbw.PREC_BF16:
+            grads += 1                                  # bf16 weight cast
+        return (0 if self.static_b is not None else 1) + grads + 1 + 1 + 2
+
+
+def agg_case(n, d, seed, b, device="cuda", mean=0.0, std=1.0):
+    """Inputs of an aggregation-only case: G [n, ld] ~ N(mean, std^2), w, Exp(1) times."""
+    ld = inputs.round_up(d, 4)
+    G = inputs.gradient_matrix(seed, n, d, ld, mean, std)
+    w = inputs.rng(seed, inputs.STREAM_INIT).standard_normal(d, dtype=np.float32)
+    times = inputs.completion_times(seed, 0, n, "shifted_exp", shift=0.0, rate=1.0)
+    return G, w, times
