@@ -168,6 +168,21 @@ int dbw_select_fastest(const double* times, int n, const int32_t* b,
                        int32_t* order, uint8_t* mask, double* tsorted,
                        int32_t* k_out, void* stream);
 
+/*
+ * Layout of the partials buffer (caller-owned scratch written by
+ * dbw_aggregate_update and read by dbw_grad_stats; public so that a caller can
+ * also assemble the sums for dbw_grad_stats itself):
+ *   int64_t header[4] = {DBW_PARTIALS_MAGIC, blocks, n, 0}
+ *   double  sums[n + 2]              reduced totals, written by dbw_grad_stats
+ *   double  vals[(n + 2) * blocks]   per-block pieces, vals[q * blocks + j]:
+ *           q < n: piece of ||g_q||^2 (0 for rows not received),
+ *           q = n: piece of the deviation sum of Eq. (10), q = n + 1: piece of ||g_t||^2.
+ * dbw_grad_stats reduces each quantity in a fixed order (256 strided fp64
+ * partial sums, then a pairwise tree), so equal buffers give equal results.
+ * A header that does not carry the magic and this call's n yields NaN sums.
+ */
+#define DBW_PARTIALS_MAGIC 0x44425750415254LL
+
 /* Bytes of the partials buffer dbw_aggregate_update needs on the current device. */
 size_t dbw_aggregate_partials_bytes(int n, int64_t d);
 

@@ -47,8 +47,12 @@ Readings of points the paper leaves open (each also listed in the design notes):
  R11 push-and-interrupt time model, see Eq. (17) above.
  R12 the statistics use the k received rows only.
  R13 ReLU'(0) = 0; numerically stable log-softmax; sampling with replacement.
- R14 bf16 operands (the two large MLPs): X and the weight matrices are rounded
-     to bf16 (round to nearest even) and everything else is fp64.
+     Where a pre-activation lies within rounding of 0 the derivative's value is a
+     decision the kernel's precision may take either way; ``worker_grads`` can
+     evaluate the other side (``relu_flip``) so that a check can accept either.
+ R14 bf16 operands (the two large MLPs): every GEMM operand -- X, the weight
+     matrices, the hidden activations and the backpropagated dZ -- is rounded to
+     bf16 (round to nearest even) as it enters a product; everything else is fp64.
 
 Scalar estimator arithmetic (F^, V^+, Eq. (11), Eq. (12), the windows, Eq. (16),
 T^_k, the ratio of Eq. (18)) is written as plain Python float operations in a
@@ -122,7 +126,7 @@ def sample_losses(widths, w, X, y, bf16=False):
     return -lsm[np.arange(A.shape[0]), np.asarray(y, dtype=np.int64)]
 
 
-def worker_grads(widths, w, X, y, n, B, bf16=False):
+def worker_grads(widths, w, X, y, n, B, bf16=False, relu_flip=None, return_preact=False):
     """Eq. (2) for every worker: G [n, d] fp64 and the minibatch mean losses [n].
 
     Rows ``i*B .. i*B+B-1`` of X / y are worker i's minibatch.  Backpropagation
@@ -130,26 +134,41 @@ def worker_grads(widths, w, X, y, n, B, bf16=False):
     the last Z.  Each worker's gradient is the mean over its own B samples, so
     dL/dZ_last = (softmax - onehot) / B and the per-worker weight gradient is
     dZ_l[i]^T A_{l-1}[i].
+
+    bf16 (R14): every GEMM operand is rounded to bf16 before it is used -- X, the
+    weight matrices, the hidden activations A_l and the backpropagated dZ_l --
+    and all arithmetic is fp64.
+
+    relu_flip (R13): optional list, one boolean [n*B, width] array per hidden
+    layer; where True the ReLU derivative takes the other one-sided value
+    (1[Z > 0] is replaced by 1[Z >= 0] semantics at that entry, i.e. the mask
+    bit is inverted).  Only meaningful where Z is within rounding of 0.
+    return_preact: also return the hidden pre-activations Z_l and their scale
+    sum_k |A_{l-1}[r,k] W_l[u,k]| + |b_l[u]| (the size a rounding error of Z is
+    relative to).
     """
+    rnd = (lambda a: bf16_round(np.asarray(a, dtype=np.float32))) if bf16 else (lambda a: a)
     w64 = np.asarray(w, dtype=np.float64)
     params = unflatten(w64, widths)
     if bf16:
-        A0 = bf16_round(X)
-        params = [(bf16_round(np.asarray(W, dtype=np.float32)), b) for (W, b) in params]
-    else:
-        A0 = np.asarray(X, dtype=np.float64)
+        params = [(rnd(W), b) for (W, b) in params]
+    A0 = rnd(np.asarray(X, dtype=np.float64))
     M = n * B
     assert A0.shape[0] == M
     L = len(params)
-    acts = [A0]          # A_0 .. A_{L-1}
-    zs = []
+    acts = [A0]          # A_0 .. A_{L-1} as the GEMMs consume them
+    zs, scales = [], []
     A = A0
     for l, (W, b) in enumerate(params):
         Z = A @ W.T + b
-        zs.append(Z)
-        A = np.maximum(Z, 0.0) if l < L - 1 else Z
         if l < L - 1:
+            zs.append(Z)
+            if return_preact:
+                scales.append(np.abs(A) @ np.abs(W).T + np.abs(b))
+            A = rnd(np.maximum(Z, 0.0))
             acts.append(A)
+        else:
+            A = Z
     logits = A
     yy = np.asarray(y, dtype=np.int64)
     lsm = _log_softmax(logits)
@@ -157,7 +176,7 @@ def worker_grads(widths, w, X, y, n, B, bf16=False):
     loss = per_sample.reshape(n, B).mean(axis=1)
     dZ = np.exp(lsm)
     dZ[np.arange(M), yy] -= 1.0
-    dZ /= B
+    dZ = rnd(dZ / B)
     layers, d = param_layout(widths)
     G = np.empty((n, d), dtype=np.float64)
     for l in range(L - 1, -1, -1):
@@ -168,13 +187,18 @@ def worker_grads(widths, w, X, y, n, B, bf16=False):
         G[:, offb:offb + fout] = dZi.sum(axis=1)
         if l > 0:
             W = params[l][0]
-            dZ = (dZ @ W) * (zs[l - 1] > 0.0)
+            live = zs[l - 1] > 0.0
+            if relu_flip is not None and relu_flip[l - 1] is not None:
+                live = live ^ relu_flip[l - 1]
+            dZ = rnd((dZ @ W) * live)
+    if return_preact:
+        return G, loss, zs, scales
     return G, loss
 
 
-def single_worker_grad(widths, w, X, y, B, bf16=False):
+def single_worker_grad(widths, w, X, y, B, bf16=False, relu_flip=None):
     """Eq. (2) for one worker only (its B rows); used for sampled checks at scale."""
-    G, loss = worker_grads(widths, w, X, y, 1, B, bf16)
+    G, loss = worker_grads(widths, w, X, y, 1, B, bf16, relu_flip)
     return G[0], loss[0]
 
 
@@ -379,6 +403,12 @@ def time_estimates(st: State):
     return [st.S[k - 1] / float(st.c) for k in range(1, st.n + 1)]
 
 
+def _ieee_div(a, b):
+    """a / b with IEEE 754 semantics (x/0 = +-inf, 0/0 = NaN) instead of a Python error."""
+    with np.errstate(divide="ignore", invalid="ignore"):
+        return float(np.float64(a) / np.float64(b))
+
+
 def choose_k(st: State, lr, beta, blind=False):
     """Eqs. (18)-(19): k_t for the iteration about to start; returns (k_t, ratio list).
 
@@ -392,7 +422,7 @@ def choose_k(st: State, lr, beta, blind=False):
             T = time_estimates(st)
             best = -math.inf
             for k in range(1, n + 1):
-                ratio[k - 1] = float(k) / T[k - 1]
+                ratio[k - 1] = _ieee_div(float(k), T[k - 1])
                 if ratio[k - 1] >= best:
                     best, kstar = ratio[k - 1], k
     else:
@@ -402,7 +432,7 @@ def choose_k(st: State, lr, beta, blind=False):
             best = -math.inf
             found = False
             for k in range(1, n + 1):
-                ratio[k - 1] = gains[k - 1] / T[k - 1]
+                ratio[k - 1] = _ieee_div(gains[k - 1], T[k - 1])
                 if gains[k - 1] > 0.0 and ratio[k - 1] >= best:
                     best, kstar, found = ratio[k - 1], k, True
             if not found:

@@ -59,7 +59,7 @@ int launch_worker_grads(int L, const int32_t* widths, int prec, const float* w, 
 //   double sums[n + 2]              reduced totals (written by dbw_grad_stats)
 //   double vals[(n + 2) * blocks]   per-block pieces, by quantity: vals[q * blocks + blk]
 //                                   q < n: ||g_q||^2, q = n: SS, q = n + 1: ||g_t||^2
-constexpr int64_t kPartialsMagic = 0x44425750415254LL;  // "DBWPART"
+constexpr int64_t kPartialsMagic = DBW_PARTIALS_MAGIC;  // "DBWPART"
 constexpr int kPartialsHeader = 4;
 
 }  // namespace dbw

@@ -23,6 +23,7 @@ CHOOSE_BLIND = 1
 FLAG_K1, FLAG_L_SKIPPED, FLAG_EMPTY_MASK, FLAG_BAD_STATE = 1, 2, 4, 8
 STAT_K, STAT_SS, STAT_GBAR_SQ, STAT_V, STAT_N, STAT_F, STAT_L, STAT_FLAGS, STAT_VCLOCK = range(9)
 STATS_LEN = 9
+PARTIALS_MAGIC = 0x44425750415254
 
 
 class DbwState(C.Structure):

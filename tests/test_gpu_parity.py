@@ -10,7 +10,8 @@ import torch
 from oracle import dbw_oracle as O
 from paper_2004_14696_gb300 import dbw, inputs, workloads
 from paper_2004_14696_gb300.pipeline import Iteration, agg_case
-from gpu_util import RTOL_BF16, RTOL_FP32, assert_close_rows, assert_close_scalar
+from gpu_util import (RTOL_BF16, RTOL_FP32, assert_close_rows, assert_close_scalar, assert_worker_grads_match,
+                      param_blocks)
 
 pytestmark = pytest.mark.gpu
 
@@ -48,19 +49,25 @@ def to_oracle_state(s: dbw.DbwState) -> O.State:
     return st
 
 
-def bits(x):
-    return np.float64(x).view(np.uint64)
+def same_f64(a, b):
+    """Bit-identical fp64 arrays, except that any NaN matches any NaN (payload and sign
+    of a NaN carry no meaning here and differ between the CUDA and numpy defaults)."""
+    a = np.atleast_1d(np.asarray(a, dtype=np.float64))
+    b = np.atleast_1d(np.asarray(b, dtype=np.float64))
+    if a.shape != b.shape:
+        return False
+    na, nb = np.isnan(a), np.isnan(b)
+    return bool(np.array_equal(na, nb) and np.array_equal(a[~na].view(np.uint64), b[~nb].view(np.uint64)))
 
 
 def assert_state_equal(g: dbw.DbwState, o: O.State):
     for f in ("t", "k_last", "c", "cntV", "cntN", "cntL", "flags", "has_last"):
         assert int(getattr(g, f)) == getattr(o, f), f
     for f in ("F_last", "F_prev", "N_last", "V_last", "vclock"):
-        assert bits(getattr(g, f)) == bits(getattr(o, f)), (f, getattr(g, f), getattr(o, f))
+        assert same_f64(getattr(g, f), getattr(o, f)), (f, getattr(g, f), getattr(o, f))
     for name in ("ringV", "ringN", "ringL"):
-        assert np.array_equal(np.array(getattr(g, name)).view(np.uint64),
-                              np.array(getattr(o, name), dtype=np.float64).view(np.uint64)), name
-    assert np.array_equal(np.array(g.S[: g.n]).view(np.uint64), np.array(o.S, dtype=np.float64).view(np.uint64))
+        assert same_f64(list(getattr(g, name)), getattr(o, name)), name
+    assert same_f64(list(g.S[: g.n]), o.S)
 
 
 # ================================================================ selection
@@ -73,7 +80,7 @@ def test_select_bit_exact(n):
             order, mask, ts = O.select_fastest(times, b)
             assert np.array_equal(got["order"], order)
             assert np.array_equal(got["mask"], mask)
-            assert np.array_equal(got["tsorted"].view(np.uint64), ts.view(np.uint64))
+            assert same_f64(got["tsorted"], ts)
             assert int(got["k"][0]) == n - b
 
 
@@ -150,72 +157,130 @@ def test_aggregate_does_not_read_padding_or_unselected_rows():
 
 
 # ================================================================ estimator
-def test_estimator_sequence_teacher_forced_bit_exact():
-    """Every iteration: GPU b_t equals the oracle's on the GPU's own state (bit for bit,
-    ratios included), and the state after dbw_grad_stats equals the oracle's bookkeeping
-    applied to the GPU's reduced sums."""
+# The estimator is checked on seeded inputs handed identically to both sides:
+# states built on the host, and partial sums made of dyadic values so that every
+# summation order gives the same exact fp64 totals.  Nothing flows from the GPU
+# into the oracle.
+def fill_state(n, D, rng):
+    """A random but consistent estimator state, as (ctypes mirror, oracle State)."""
+    g = dbw.DbwState()
+    o = O.State(n=n, D=D)
+    g.n, g.D = n, D
+    vals = dict(t=int(rng.integers(0, 30)), k_last=int(rng.integers(1, n + 1)), c=int(rng.integers(0, 12)),
+                cntV=int(rng.integers(0, 3 * D)), cntN=int(rng.integers(0, 3 * D)),
+                cntL=int(rng.integers(0, 3 * D)), has_last=int(rng.integers(0, 2)))
+    if rng.random() < 0.7:
+        vals["cntV"] = max(vals["cntV"], 1)
+        vals["cntN"] = max(vals["cntN"], 1)
+        vals["cntL"] = max(vals["cntL"], 1)
+        vals["c"] = max(vals["c"], 1)
+    for k, v in vals.items():
+        setattr(g, k, v)
+        setattr(o, k, v)
+    F_prev = float(rng.uniform(0.5, 3.0))
+    F_last = F_prev * float(rng.choice([0.98, 1.0, 1.01, 1.02, 1.3]))
+    fl = dict(F_last=F_last, F_prev=F_prev, N_last=float(rng.uniform(0, 2)), V_last=float(rng.uniform(0, 9)),
+              vclock=float(rng.uniform(0, 100)))
+    for k, v in fl.items():
+        setattr(g, k, v)
+        setattr(o, k, v)
+    ringV = rng.uniform(0, 10, O.DMAX) * rng.choice([0.0, 1.0], O.DMAX, p=[0.1, 0.9])
+    ringN = rng.uniform(0, 2, O.DMAX) * rng.choice([0.0, 1.0], O.DMAX, p=[0.2, 0.8])
+    ringL = rng.uniform(-2, 40, O.DMAX)
+    for name, arr in (("ringV", ringV), ("ringN", ringN), ("ringL", ringL)):
+        getattr(g, name)[:] = arr.tolist()
+        setattr(o, name, arr.tolist())
+    times = np.sort(np.round(rng.exponential(size=n), 2)) * max(vals["c"], 1)
+    S = np.zeros(dbw.NMAX)
+    S[:n] = times
+    g.S[:] = S.tolist()
+    o.S = times.tolist()
+    return g, o
+
+
+def test_choose_b_bit_exact_on_seeded_states():
+    rng = np.random.default_rng(2024)
+    b = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for trial in range(400):
+        n = int(rng.choice([1, 2, 3, 7, 16, 64, 256, 1024]))
+        D = int(rng.choice([1, 3, 5, 64]))
+        g, o = fill_state(n, D, rng)
+        lr = float(rng.choice([0.01, 0.05, 0.1]))
+        beta = float(rng.choice([1.0, 1.01, 1.05]))
+        blind = bool(rng.random() < 0.15)
+        state = torch.empty(dbw.STATE_BYTES, dtype=torch.uint8, device="cuda")
+        dbw.write_state(state, g)
+        ratio = torch.empty(n, dtype=torch.float64, device="cuda")
+        dbw.dbw_choose_b(state, lr, beta, b, ratio, flags=dbw.CHOOSE_BLIND if blind else 0)
+        torch.cuda.synchronize()
+        k, r = O.choose_k(o, lr, beta, blind=blind)
+        assert n - int(b.item()) == k, trial
+        assert same_f64(ratio.cpu().numpy(), r), trial
+        assert dbw.read_state(state).k_next == k
+
+
+def seeded_partials(n, blocks, SS, g2, rows, device="cuda"):
+    """A partials buffer (layout of include/dbw.h) whose per-block pieces sum exactly to SS, g2, rows."""
+    vals = np.zeros((n + 2, blocks))
+    for q, total in list(enumerate(rows)) + [(n, SS), (n + 1, g2)]:
+        units = int(round(total * 1024))           # dyadic: multiples of 2^-10
+        cuts = np.sort(np.random.default_rng(q).integers(0, units + 1, blocks - 1)) if units > 0 else \
+            np.zeros(blocks - 1, dtype=np.int64)
+        parts = np.diff(np.concatenate([[0], cuts, [units]]))
+        vals[q] = parts / 1024.0
+    head = np.array([dbw.PARTIALS_MAGIC, blocks, n, 0], dtype=np.int64).view(np.uint8)
+    body = np.concatenate([np.zeros(n + 2), vals.ravel()]).view(np.uint8)
+    return dev(np.concatenate([head, body]))
+
+
+def test_estimator_trajectory_bit_exact():
+    """60 DBW iterations of the estimator alone, both sides fed the same seeded sums,
+    losses and times: every b_t, ratio vector and state is identical bit for bit, and
+    k_t moves the way Sect. 4 describes (small while ||grad F||^2 dominates, growing
+    as it falls), with the loss-increase guard tripping on the loss bumps."""
     n, d, D, lr, beta = 16, 3001, 5, 0.05, 1.01
     rng = np.random.default_rng(42)
     state = dbw.new_state(n, D)
+    ost = O.State(n=n, D=D)
     b = torch.zeros(1, dtype=torch.int32, device="cuda")
     ratio = torch.empty(n, dtype=torch.float64, device="cuda")
-    part = torch.empty(dbw.dbw_aggregate_partials_bytes(n, d), dtype=torch.uint8, device="cuda")
     stats = torch.empty(dbw.STATS_LEN, dtype=torch.float64, device="cuda")
-    w = dev(rng.standard_normal(d).astype(np.float32))
-    decisions = set()
+    rn = torch.empty(n, dtype=torch.float64, device="cuda")
+    ks = []
     F, prev = 50.0, None
     for t in range(60):
-        ost = to_oracle_state(dbw.read_state(state))
         dbw.dbw_choose_b(state, lr, beta, b, ratio)
         torch.cuda.synchronize()
-        k_or, ratio_or = O.choose_k(ost, lr, beta)
-        assert n - int(b.item()) == k_or, t
-        assert np.array_equal(ratio.cpu().numpy().view(np.uint64), np.array(ratio_or).view(np.uint64)), t
-        decisions.add(k_or)
-        # gradients whose mean shrinks over time (N falls towards V/k, so k_t should grow);
-        # losses fall by the gain Eq. (9) predicts for L = 5, with a bump every 9 iterations
-        # that trips the guard of Eq. (19)
+        k, r = O.choose_k(ost, lr, beta)
+        assert n - int(b.item()) == k, t
+        assert same_f64(ratio.cpu().numpy(), r), t
+        ks.append(k)
+        # sums of k rows ~ N(mu_t, 1) in d columns: SS ~ (k-1) d, ||g_t||^2 ~ d mu_t^2 + d / k
         mu = 0.5 * math.exp(-t / 12.0)
-        G = (mu + rng.standard_normal((n, d))).astype(np.float32)
-        G = np.pad(G, ((0, 0), (0, inputs.round_up(d, 4) - d)))
-        times = np.round(1.0 + rng.exponential(size=n), 1)     # ties happen
+        SS = (k - 1) * d * float(rng.uniform(0.95, 1.05))
+        g2 = d * mu * mu + d / k * float(rng.uniform(0.9, 1.1))
+        times = np.round(1.0 + rng.exponential(size=n), 1)
         if prev is not None:
             N, V, kk = prev
             F = F - ((lr - 5 * lr * lr / 2) * N - (5 * lr * lr / 2) * V / kk) + (0.5 if t % 9 == 4 else 0.0)
         loss = (F + 0.01 * rng.standard_normal(n)).astype(np.float32)
-        sel = gpu_select(times, int(b.item()))
-        dbw.dbw_aggregate_update(dev(G), n, d, dev(sel["mask"]), lr, w, part)
-        dbw.dbw_grad_stats(part, n, dev(sel["mask"]), dev(loss), dev(sel["tsorted"]), lr, state, stats)
+        sel = gpu_select(times, n - k)
+        _, mask, ts = O.select_fastest(times, n - k)
+        assert np.array_equal(sel["mask"], mask)
+        rows = [float(rng.integers(1, 1 << 20)) / 1024.0 if mask[j] else 0.0 for j in range(n)]
+        SSq, g2q = round(SS * 1024) / 1024.0, round(g2 * 1024) / 1024.0
+        part = seeded_partials(n, 3, SSq, g2q, rows)
+        dbw.dbw_grad_stats(part, n, dev(mask), dev(loss), dev(ts), lr, state, stats, rn)
         torch.cuda.synchronize()
-        s = stats.cpu().numpy()
-        k = int(s[dbw.STAT_K])
-        prev = (float(s[dbw.STAT_N]), float(s[dbw.STAT_V]), k) if k >= 2 else None
-        O.record_iteration(ost, k, float(s[dbw.STAT_SS]), float(s[dbw.STAT_GBAR_SQ]), loss,
-                           sel["mask"], sel["tsorted"], lr)
+        rec = O.record_iteration(ost, k, SSq, g2q, loss, mask, ts, lr)
         assert_state_equal(dbw.read_state(state), ost)
-    assert len(decisions) > 5, decisions      # the estimator actually moved
-
-
-def test_blind_variant_bit_exact():
-    n = 12
-    state = dbw.new_state(n, 5)
-    part = torch.empty(dbw.dbw_aggregate_partials_bytes(n, 64), dtype=torch.uint8, device="cuda")
-    b = torch.zeros(1, dtype=torch.int32, device="cuda")
-    ratio = torch.empty(n, dtype=torch.float64, device="cuda")
-    rng = np.random.default_rng(1)
-    w = dev(np.zeros(64, np.float32))
-    for t in range(5):
-        times = 1.0 + rng.exponential(size=n)
-        sel = gpu_select(times, 0)
-        G = rng.standard_normal((n, 64)).astype(np.float32)
-        dbw.dbw_aggregate_update(dev(G), n, 64, dev(sel["mask"]), 0.1, w, part)
-        dbw.dbw_grad_stats(part, n, dev(sel["mask"]), dev(np.ones(n, np.float32)), dev(sel["tsorted"]), 0.1, state)
-    ost = to_oracle_state(dbw.read_state(state))
-    dbw.dbw_choose_b(state, 0.1, 1.01, b, ratio, flags=dbw.CHOOSE_BLIND)
-    torch.cuda.synchronize()
-    k, r = O.choose_k(ost, 0.1, 1.01, blind=True)
-    assert n - int(b.item()) == k
-    assert np.array_equal(ratio.cpu().numpy().view(np.uint64), np.array(r).view(np.uint64))
+        st = stats.cpu().numpy()
+        for key, idx in (("V", dbw.STAT_V), ("N", dbw.STAT_N), ("F", dbw.STAT_F), ("L", dbw.STAT_L),
+                         ("SS", dbw.STAT_SS), ("gbar_sq", dbw.STAT_GBAR_SQ), ("vclock", dbw.STAT_VCLOCK)):
+            assert same_f64(st[idx], rec[key]), (t, key)
+        assert same_f64(rn.cpu().numpy(), [rows[j] if mask[j] else math.nan for j in range(n)])
+        prev = (rec["N"], rec["V"], k) if k >= 2 else None
+    assert len(set(ks)) > 5 and min(ks) < 8 and ks[-1] == n, ks
 
 
 def test_empty_mask_and_bad_state_raise_flags_without_fault():
@@ -260,10 +325,10 @@ def grads_case(wl, t=0):
 def test_worker_grads_parity_full(wl):
     it, idx = grads_case(wl)
     pool, labels, w = it.pool.cpu().numpy(), it.labels.cpu().numpy(), it.w.cpu().numpy()
-    G, loss = O.worker_grads(wl.widths, w, pool[idx], labels[idx], wl.n, wl.B, bf16=wl.prec == workloads.PREC_BF16)
-    rtol = RTOL_BF16 if wl.prec == workloads.PREC_BF16 else RTOL_FP32
-    assert_close_rows(it.G.cpu().numpy()[:, :wl.d], G, rtol, "G")
-    assert_close_rows(it.loss.cpu().numpy(), loss, rtol, "loss")
+    bf16 = wl.prec == workloads.PREC_BF16
+    rtol = RTOL_BF16 if bf16 else RTOL_FP32
+    assert_worker_grads_match(it.G.cpu().numpy()[:, :wl.d], it.loss.cpu().numpy(), wl.widths, w, pool[idx],
+                              labels[idx], wl.B, bf16, range(wl.n), rtol)
 
 
 @pytest.mark.parametrize("wl", [workloads.MLP3072], ids=lambda w: w.key)
@@ -271,11 +336,10 @@ def test_worker_grads_parity_sampled_workers(wl):
     """Full-size bf16 config: the oracle recomputes a few sampled workers from their own minibatch."""
     it, idx = grads_case(wl)
     pool, labels, w = it.pool.cpu().numpy(), it.labels.cpu().numpy(), it.w.cpu().numpy()
-    for i in (0, wl.n - 1, 37):
-        rows = idx[i * wl.B:(i + 1) * wl.B]
-        g, l = O.single_worker_grad(wl.widths, w, pool[rows], labels[rows], wl.B, bf16=True)
-        assert_close_rows(it.G[i, :wl.d].cpu().numpy(), g, RTOL_BF16, f"G row {i}")
-        assert_close_scalar(it.loss[i].item(), l, RTOL_BF16, f"loss {i}")
+    workers = (0, 37, wl.n - 1)
+    rows = {i: it.G[i, :wl.d].cpu().numpy() for i in workers}
+    assert_worker_grads_match(rows, it.loss.cpu().numpy(), wl.widths, w, pool[idx], labels[idx], wl.B, True,
+                              workers, RTOL_BF16)
 
 
 def test_bad_sample_index_poisons_only_that_worker():
@@ -293,32 +357,66 @@ def test_bad_sample_index_poisons_only_that_worker():
 
 
 # ================================================================ whole iterations
+def decision_margin(st: O.State, lr, beta):
+    """How far the oracle's b_t is from flipping: the relative gap between the best and
+    the runner-up ratio of Eq. (18), and of the guard comparison of Eq. (19)."""
+    gains = O.gain_estimates(st, lr)
+    gaps = [math.inf]
+    if gains is not None:
+        T = O.time_estimates(st)
+        r = sorted((g / t for g, t in zip(gains, T) if g > 0), reverse=True)
+        if len(r) >= 2:
+            gaps.append((r[0] - r[1]) / abs(r[0]))
+        gaps.append(min(abs(g) for g in gains) / max(abs(g) for g in gains) if max(abs(g) for g in gains) > 0
+                    else math.inf)
+    if st.t >= 2 and st.k_last < st.n:
+        gaps.append(abs(st.F_last - beta * st.F_prev) / abs(st.F_last))
+    return min(gaps)
+
+
 @pytest.mark.parametrize("wl,iters", [(workloads.MLP784, 6), (SMALL_BF16, 8)], ids=["mlp784", "small_bf16"])
-def test_dbw_iterations_teacher_forced(wl, iters):
-    """Whole DBW iterations through the pipeline; each is compared with the oracle
-    started from the GPU's own w_t and state (teacher forcing)."""
+def test_dbw_iterations_independent(wl, iters):
+    """Whole DBW iterations: the GPU pipeline and the oracle each run their own
+    trajectory from the same seeds.  b_t must agree exactly unless the oracle's own
+    decision is within 1e-3 of flipping (then both choices are valid at fp32 input
+    precision and the trajectories part; the comparison stops there)."""
     it = Iteration(wl, keep_gbar=True)
     pool, labels = it.pool.cpu().numpy(), it.labels.cpu().numpy()
     bf16 = wl.prec == workloads.PREC_BF16
     rtol = RTOL_BF16 if bf16 else RTOL_FP32
+    ost = O.State(n=wl.n, D=wl.D)
+    w_or = inputs.kaiming_uniform_params(wl.seed, wl.widths).astype(np.float64)
+    compared = 0
     for t in range(iters):
-        w0 = it.w.cpu().numpy().copy()
-        ost = to_oracle_state(dbw.read_state(it.state))
         idx, times = it.host_inputs(t)
+        margin = decision_margin(ost, wl.lr, wl.beta)
+        k_or, _ = O.choose_k(ost, wl.lr, wl.beta)
         it.load_inputs(t)
         it.step()
         torch.cuda.synchronize()
-        k_or, _ = O.choose_k(ost, wl.lr, wl.beta)
         b = int(it.b.item())
-        assert wl.n - b == k_or, t
-        ref = O.step(ost, wl.widths, w0, pool[idx], labels[idx], times, wl.B, wl.lr, wl.beta, bf16=bf16, b=b)
-        assert np.array_equal(it.mask.cpu().numpy(), ref["mask"])
-        assert np.array_equal(it.order.cpu().numpy(), ref["order"])
-        assert_close_rows(it.G.cpu().numpy()[:, :wl.d], ref["G"], rtol, "G")
-        assert_close_rows(it.gbar.cpu().numpy(), ref["gbar"], rtol, "g_t")
-        assert_close_rows(it.w.cpu().numpy(), ref["w"], rtol, "w")
+        if wl.n - b != k_or:
+            assert margin < 1e-3, (t, b, k_or, margin)
+            break
+        blocks = param_blocks(wl.widths)
+        matched = assert_worker_grads_match(it.G.cpu().numpy()[:, :wl.d], it.loss.cpu().numpy(), wl.widths, w_or,
+                                            pool[idx], labels[idx], wl.B, bf16, range(wl.n), rtol)
+        G_ref = np.stack([matched[i][0] for i in range(wl.n)])
+        loss_ref = np.array([matched[i][1] for i in range(wl.n)])
+        order, mask, ts = O.select_fastest(times, b)
+        assert np.array_equal(it.mask.cpu().numpy(), mask)
+        assert np.array_equal(it.order.cpu().numpy(), order)
+        gbar = O.aggregate(G_ref, mask)
+        w_new = O.sgd_update(w_or, gbar, wl.lr)
+        SS = O.deviation_sumsq(G_ref, mask, gbar)
+        rec = O.record_iteration(ost, wl.n - b, SS, float(gbar @ gbar), loss_ref, mask, ts, wl.lr)
+        assert_close_rows(it.gbar.cpu().numpy(), gbar, rtol, "g_t", blocks)
+        assert_close_rows(it.w.cpu().numpy(), w_new, rtol, "w", blocks)
         s = it.stats.cpu().numpy()
-        assert_close_scalar(s[dbw.STAT_GBAR_SQ], ref["gbar_sq"], rtol, "||g_t||^2")
-        if ref["k"] >= 2:
-            assert_close_scalar(s[dbw.STAT_SS], ref["SS"], rtol, "SS")
-        assert_close_scalar(s[dbw.STAT_F], ref["F"], rtol, "F")
+        assert_close_scalar(s[dbw.STAT_GBAR_SQ], rec["gbar_sq"], rtol, "||g_t||^2")
+        if rec["k"] >= 2:
+            assert_close_scalar(s[dbw.STAT_SS], rec["SS"], rtol, "SS")
+        assert_close_scalar(s[dbw.STAT_F], rec["F"], rtol, "F")
+        w_or = w_new
+        compared += 1
+    assert compared >= 3

@@ -203,3 +203,10 @@ def test_planted_sign_error_in_gain_is_caught(monkeypatch, paper):
     monkeypatch.setattr(O, "gain_estimates", flipped)
     with pytest.raises(AssertionError):
         test_equal_times_choose_all_workers(paper)
+
+
+def test_zero_time_estimate_follows_ieee_division():
+    """A time estimate of 0 gives an infinite ratio (IEEE), which Eq. (18) then prefers."""
+    st = _state_with(4, V=1.0, N=1.0, L=1.0, T=[0.0, 1.0, 2.0, 3.0])
+    k, ratio = O.choose_k(st, 0.05, 1.01)
+    assert ratio[0] == math.inf and k == 1

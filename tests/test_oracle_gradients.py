@@ -79,17 +79,54 @@ def test_bf16_round_matches_torch_conversion():
     assert O.bf16_round(np.float32([1.01171875]))[0] == 1.015625
 
 
-def test_bf16_mode_is_fp64_math_on_rounded_operands():
-    widths, n, B = (6, 5, 3), 2, 3
+def test_bf16_mode_rounds_every_gemm_operand():
+    """bf16 mode stays within bf16 precision of the fp64 gradient, differs from the
+    fp64 computation on merely pre-rounded X and W (so the hidden operands really
+    are rounded), and on a one-layer model equals the closed form on rounded X, W, dZ."""
+    widths, n, B = (16, 12, 5), 3, 8
     w, X, y = _problem(widths, n, B, 4)
     G16, l16 = O.worker_grads(widths, w, X, y, n, B, bf16=True)
+    G64, l64 = O.worker_grads(widths, w, X, y, n, B)
+    # no ReLU (softmax regression): bf16 rounding only perturbs, by about 2^-8 relative
+    ws, Xs, ys = _problem((64, 10), n, B, 7)
+    Gs16, _ = O.worker_grads((64, 10), ws, Xs, ys, n, B, bf16=True)
+    Gs64, _ = O.worker_grads((64, 10), ws, Xs, ys, n, B)
+    assert np.linalg.norm(Gs16 - Gs64) <= 0.02 * np.linalg.norm(Gs64)
+    assert np.all(np.abs(l16 - l64) <= 0.02 * np.abs(l64))
     layers, _ = O.param_layout(widths)
     wr = w.astype(np.float64).copy()
     for (offW, fout, fin, offb) in layers:
         wr[offW:offW + fout * fin] = O.bf16_round(w[offW:offW + fout * fin])
-    G64, l64 = O.worker_grads(widths, wr, O.bf16_round(X), y, n, B)
-    np.testing.assert_allclose(G16, G64, rtol=1e-13, atol=1e-15)
-    np.testing.assert_allclose(l16, l64, rtol=1e-13)
+    Gpre, _ = O.worker_grads(widths, wr, O.bf16_round(X), y, n, B)
+    assert not np.array_equal(G16, Gpre)
+    # one layer: g_W = dZ^T X with dZ = bf16((p - e_y) / B), X and W rounded
+    widths1 = (16, 5)
+    w1, X1, y1 = _problem(widths1, 1, B, 5)
+    G1, _ = O.worker_grads(widths1, w1, X1, y1, 1, B, bf16=True)
+    Wr = O.bf16_round(w1[:80]).reshape(5, 16)
+    Xr = O.bf16_round(X1)
+    z = Xr @ Wr.T + w1[80:].astype(np.float64)
+    p = np.exp(z - z.max(1, keepdims=True))
+    p /= p.sum(1, keepdims=True)
+    dZ = O.bf16_round(((p - np.eye(5)[y1]) / B).astype(np.float32))
+    np.testing.assert_allclose(G1[0, :80], (dZ.T @ Xr).ravel(), rtol=1e-13, atol=1e-16)
+    np.testing.assert_allclose(G1[0, 80:], dZ.sum(0), rtol=1e-13, atol=1e-16)
+
+
+def test_relu_flip_changes_only_the_flipped_unit_and_below():
+    widths, n, B = (6, 5, 4), 1, 3
+    w, X, y = _problem(widths, n, B, 6)
+    G, _, zs, scales = O.worker_grads(widths, w, X, y, n, B, return_preact=True)
+    assert zs[0].shape == (3, 5) and np.all(scales[0] >= np.abs(zs[0]))
+    flip = np.zeros((3, 5), dtype=bool)
+    flip[1, 2] = True
+    Gf, _ = O.worker_grads(widths, w, X, y, n, B, relu_flip=[flip])
+    layers, _ = O.param_layout(widths)
+    offW, fout, fin, offb = layers[0]
+    changed = np.flatnonzero(G[0] != Gf[0])
+    rows = set((c - offW) // fin for c in changed if c < offb)
+    assert rows <= {2}                                   # only unit 2's weight row (and its bias)
+    assert all(c < layers[1][0] for c in changed)        # the output layer is untouched
 
 
 def test_single_worker_grad_equals_row_of_batch():
