@@ -206,6 +206,36 @@ int dbw_aggregate_update(const float* G, int64_t ld, int n, int64_t d,
                          const uint8_t* mask, float lr, float* w, float* gbar,
                          double* partials, size_t partials_bytes, void* stream);
 
+/*
+ * dbw_aggregate_update_noalloc: the same fused aggregation as
+ * dbw_aggregate_update, for callers that cannot provide scratch memory.  The
+ * paper has no counterpart to this call; it exists for integration.
+ *
+ * Some callers may not allocate device memory at all: a plugin inside a host
+ * application that owns the whole GPU memory budget and hands out only the
+ * tensors to work on, or a latency-critical loop in which cudaMalloc (which can
+ * synchronise the device) is not acceptable.  This call needs no scratch from
+ * them and allocates nothing: its per-block partial sums go to one built-in
+ * device array of DBW_NOALLOC_SCRATCH_BYTES that every GPU loading the library
+ * holds until the process exits.  That is enough for n <= 1024 on a 152-SM GB300;
+ * if (n, d) would need more on the current device the call returns DBW_EINVAL
+ * (use dbw_aggregate_update with caller memory instead).
+ *
+ * The first call on each device looks up the array's device address (the
+ * runtime's cudaGetSymbolAddress, with that device current) and caches it; make
+ * that first call before any stream capture begins.  All calls on a device
+ * share the array: calls whose GPU work overlaps (unordered streams) race and
+ * corrupt each other's sums.  Nothing in the array needs to start at zero.
+ *
+ *  G, ld, n, d, mask, lr, w, gbar   as for dbw_aggregate_update.
+ *  sums_out  [n + 2] fp64 device out: sums_out[j] = ||g_j||^2 for received rows
+ *            (0 otherwise), sums_out[n] = the deviation sum of Eq. (10),
+ *            sums_out[n + 1] = ||g_t||^2 -- the totals dbw_grad_stats would form.
+ */
+#define DBW_NOALLOC_SCRATCH_BYTES ((size_t)4 << 20)
+int dbw_aggregate_update_noalloc(const float* G, int64_t ld, int n, int64_t d, const uint8_t* mask, float lr,
+                                 float* w, float* gbar, double* sums_out, void* stream);
+
 /* Initialise a device dbw_state for n workers and window D (k_0 = n). */
 int dbw_state_init(dbw_state* state, int n, int D, void* stream);
 

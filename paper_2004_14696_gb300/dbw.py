@@ -61,6 +61,7 @@ _SIGS = {
     "dbw_select_fastest": (_i32, [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp]),
     "dbw_aggregate_partials_bytes": (_sz, [_i32, _i64]),
     "dbw_aggregate_update": (_i32, [_vp, _i64, _i32, _i64, _vp, _f32, _vp, _vp, _vp, _sz, _vp]),
+    "dbw_aggregate_update_noalloc": (_i32, [_vp, _i64, _i32, _i64, _vp, _f32, _vp, _vp, _vp, _vp]),
     "dbw_state_init": (_i32, [_vp, _i32, _i32, _vp]),
     "dbw_grad_stats": (_i32, [_vp, _i32, _vp, _vp, _vp, _f64, _vp, _vp, _vp, _vp]),
     "dbw_choose_b": (_i32, [_vp, _f64, _f64, _i32, _vp, _vp, _vp]),
@@ -155,6 +156,16 @@ def dbw_aggregate_update(G, n, d, mask, lr, w, partials, gbar=None, stream=None)
         _ptr(w, torch.float32, "w"), _ptr(gbar, torch.float32, "gbar", nullable=True),
         _ptr(partials, torch.uint8, "partials"), partials.numel(), _stream(stream))
     _check("dbw_aggregate_update", rc)
+
+
+def dbw_aggregate_update_noalloc(G, n, d, mask, lr, w, sums_out, gbar=None, stream=None):
+    """dbw_aggregate_update without caller scratch (for callers that cannot allocate);
+    writes the reduced totals to sums_out [n + 2] fp64."""
+    rc = lib().dbw_aggregate_update_noalloc(
+        _ptr(G, torch.float32, "G"), G.shape[1], n, d, _ptr(mask, torch.uint8, "mask"), float(lr),
+        _ptr(w, torch.float32, "w"), _ptr(gbar, torch.float32, "gbar", nullable=True),
+        _ptr(sums_out, torch.float64, "sums_out"), _stream(stream))
+    _check("dbw_aggregate_update_noalloc", rc)
 
 
 def dbw_state_init(state, n, D, stream=None):
