@@ -1,0 +1,123 @@
+"""Run single pieces of the DBW iteration on chosen sizes, for timing and ncu captures.
+
+    python -m paper_2004_14696_gb300.profile_case aggregate --n 64 --d 4000000 --b 16 --reps 3
+    python -m paper_2004_14696_gb300.profile_case sweep            # the aggregation-only sweep
+    python -m paper_2004_14696_gb300.profile_case grads --workload mlp4096x3-1000_n256_B32 --reps 3
+
+Each prints one JSON line per case with CUDA-event times (on the launching
+stream, after warm-up).  Large gradient matrices are filled on the device with
+torch's seeded normal generator (input generation only); times come from the
+same seeded host models as everywhere else.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+
+import numpy as np
+import torch
+
+from . import dbw, inputs, workloads
+from .pipeline import Iteration
+
+
+def _peak_hbm():
+    path = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return json.load(f)["hbm_gbs"], "measured"
+    return 6800.0, "fallback"
+
+
+def aggregate_case(n, d, b, reps, seed=2004146963, warmup=2):
+    ld = inputs.round_up(d, 4)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed + n)
+    G = torch.randn((n, ld), generator=g, device="cuda", dtype=torch.float32)
+    w = torch.randn(d, generator=g, device="cuda", dtype=torch.float32)
+    times = torch.from_numpy(inputs.completion_times(seed, 0, n, "shifted_exp", shift=0.0, rate=1.0)).cuda()
+    bt = torch.tensor([b], dtype=torch.int32, device="cuda")
+    order = torch.empty(n, dtype=torch.int32, device="cuda")
+    mask = torch.empty(n, dtype=torch.uint8, device="cuda")
+    ts = torch.empty(n, dtype=torch.float64, device="cuda")
+    dbw.dbw_select_fastest(times, bt, order, mask, ts)
+    part = torch.empty(dbw.dbw_aggregate_partials_bytes(n, d), dtype=torch.uint8, device="cuda")
+    for _ in range(warmup):
+        dbw.dbw_aggregate_update(G, n, d, mask, 1e-3, w, part)
+    st = torch.cuda.current_stream()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    torch.cuda.synchronize()
+    for e0, e1 in evs:
+        e0.record(st)
+        dbw.dbw_aggregate_update(G, n, d, mask, 1e-3, w, part)
+        e1.record(st)
+    torch.cuda.synchronize()
+    ms = [e0.elapsed_time(e1) for e0, e1 in evs]
+    k = n - b
+    nbytes = (k * d + 2 * d) * 4
+    avg = float(np.mean(ms))
+    peak, src = _peak_hbm()
+    gbs = nbytes / (avg * 1e-3) / 1e9
+    l2_note = "G > L2" if n * ld * 4 > 129e6 else "G fits in L2 (reads may hit L2)"
+    return {"case": "aggregate", "n": n, "d": d, "b": b, "k": k, "G_bytes": n * ld * 4, "bytes": nbytes,
+            "ms": avg, "ms_min": min(ms), "GB_s": gbs, "frac_of_peak": gbs / peak, "peak_GB_s": peak,
+            "peak_source": src, "reps": reps, "l2": l2_note}
+
+
+def grads_case(key, reps, warmup=2):
+    wl = workloads.ALL[key]
+    it = Iteration(wl, static_b=0)
+    it.load_inputs(0)
+    for _ in range(warmup):
+        dbw.dbw_worker_grads(wl.widths, wl.prec, it.w, it.pool, it.labels, it.idx, wl.n, wl.B, it.G, it.loss, it.ws)
+    st = torch.cuda.current_stream()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    torch.cuda.synchronize()
+    for e0, e1 in evs:
+        e0.record(st)
+        dbw.dbw_worker_grads(wl.widths, wl.prec, it.w, it.pool, it.labels, it.idx, wl.n, wl.B, it.G, it.loss, it.ws)
+        e1.record(st)
+    torch.cuda.synchronize()
+    ms = [e0.elapsed_time(e1) for e0, e1 in evs]
+    M = wl.n * wl.B
+    flop = 0
+    for l in range(len(wl.widths) - 1):
+        flop += 4 * M * wl.widths[l] * wl.widths[l + 1] + (2 * M * wl.widths[l] * wl.widths[l + 1] if l else 0)
+    avg = float(np.mean(ms))
+    return {"case": "worker_grads", "workload": key, "ms": avg, "ms_min": min(ms), "flop": flop,
+            "TFLOP_s": flop / (avg * 1e-3) / 1e12, "G_write_GB_s": wl.n * wl.ld * 4 / (avg * 1e-3) / 1e9}
+
+
+def main(argv=None):
+    p = argparse.ArgumentParser()
+    sub = p.add_subparsers(dest="cmd", required=True)
+    a = sub.add_parser("aggregate")
+    a.add_argument("--n", type=int, default=64)
+    a.add_argument("--d", type=int, default=4_000_000)
+    a.add_argument("--b", type=int, default=16)
+    a.add_argument("--reps", type=int, default=5)
+    s = sub.add_parser("sweep")
+    s.add_argument("--reps", type=int, default=10)
+    s.add_argument("--max-bytes", type=float, default=float(workloads.AGG_MAX_BYTES))
+    gr = sub.add_parser("grads")
+    gr.add_argument("--workload", default=workloads.MLP4096.key, choices=list(workloads.ALL))
+    gr.add_argument("--reps", type=int, default=3)
+    args = p.parse_args(argv)
+    torch.cuda.set_device(0)
+    if args.cmd == "aggregate":
+        print(json.dumps(aggregate_case(args.n, args.d, args.b, args.reps)), flush=True)
+    elif args.cmd == "sweep":
+        for n in workloads.AGG_NS:
+            for d in workloads.AGG_DS:
+                if n * inputs.round_up(d, 4) * 4 > args.max_bytes:
+                    continue
+                for b in sorted({0, n // 4}):
+                    print(json.dumps(aggregate_case(n, d, b, args.reps)), flush=True)
+                    torch.cuda.empty_cache()
+    else:
+        print(json.dumps(grads_case(args.workload, args.reps)), flush=True)
+
+
+if __name__ == "__main__":
+    main()
