@@ -140,7 +140,12 @@ size_t dbw_worker_grads_workspace_bytes(int num_layers, const int32_t* widths, i
  *          aligned.  Columns d..ld-1 are not written.
  *  loss    [n] fp32 output: each worker's minibatch mean loss (Sect. 3.1, F^_t).
  *  ws      workspace of ws_bytes >= dbw_worker_grads_workspace_bytes(...),
- *          256-byte aligned; contents are scratch.
+ *          256-byte aligned; contents are scratch, except that its first 4
+ *          bytes hold a status word once the call's device work is done: 0 on
+ *          success, bit 0 set if a tensor-core pipeline wait timed out (it is
+ *          bounded, never a hang), in which case G and loss are undefined.
+ *  Path: with prec = DBW_PREC_BF16 and B a multiple of 32 the GEMMs run on
+ *  the tcgen05 tensor cores; otherwise on fp32 FFMA (SIMT) tiles.
  *  prec    DBW_PREC_FP32 or DBW_PREC_BF16.
  */
 int dbw_worker_grads(int num_layers, const int32_t* widths, int prec,
@@ -149,6 +154,18 @@ int dbw_worker_grads(int num_layers, const int32_t* widths, int prec,
                      const int32_t* idx, int n, int B,
                      float* G, int64_t ld, float* loss,
                      void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Where dbw_worker_grads leaves the input activations of layer ``layer``
+ * (1 <= layer < num_layers: the hidden activations A = ReLU(Z) of the layer
+ * below) inside ``ws``: *offset bytes from ws, rows of *ld elements of
+ * *elem_bytes bytes (4 = fp32, 2 = bf16), one row per sample, M = n*B rows.
+ * Valid once a call's device work is done, until ws is used again.  A hidden
+ * unit's ReLU derivative is 1[A > 0], so this is also where a caller reads
+ * which units were active.  Host only; DBW_EINVAL for an invalid argument.
+ */
+int dbw_worker_grads_activations(int num_layers, const int32_t* widths, int n, int B, int prec, int layer,
+                                 size_t* offset, int64_t* ld, int* elem_bytes);
 
 /*
  * Eq. (4): the PS waits for the first k = n - b gradients.

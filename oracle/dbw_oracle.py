@@ -126,7 +126,7 @@ def sample_losses(widths, w, X, y, bf16=False):
     return -lsm[np.arange(A.shape[0]), np.asarray(y, dtype=np.int64)]
 
 
-def worker_grads(widths, w, X, y, n, B, bf16=False, relu_flip=None, return_preact=False):
+def worker_grads(widths, w, X, y, n, B, bf16=False, relu_flip=None, return_preact=False, return_magnitude=False):
     """Eq. (2) for every worker: G [n, d] fp64 and the minibatch mean losses [n].
 
     Rows ``i*B .. i*B+B-1`` of X / y are worker i's minibatch.  Backpropagation
@@ -146,6 +146,10 @@ def worker_grads(widths, w, X, y, n, B, bf16=False, relu_flip=None, return_preac
     return_preact: also return the hidden pre-activations Z_l and their scale
     sum_k |A_{l-1}[r,k] W_l[u,k]| + |b_l[u]| (the size a rounding error of Z is
     relative to).
+    return_magnitude: also return, for every entry of G, the sum of the absolute
+    values of the products it is made of (|dZ_l|^T |A_{l-1}| for weights, the sum
+    of |dZ_l| for biases): the scale a floating-point error of that entry is
+    relative to.  Returned last.
     """
     rnd = (lambda a: bf16_round(np.asarray(a, dtype=np.float32))) if bf16 else (lambda a: a)
     w64 = np.asarray(w, dtype=np.float64)
@@ -179,21 +183,28 @@ def worker_grads(widths, w, X, y, n, B, bf16=False, relu_flip=None, return_preac
     dZ = rnd(dZ / B)
     layers, d = param_layout(widths)
     G = np.empty((n, d), dtype=np.float64)
+    Gmag = np.empty((n, d), dtype=np.float64) if return_magnitude else None
     for l in range(L - 1, -1, -1):
         offW, fout, fin, offb = layers[l]
         Ain = acts[l].reshape(n, B, fin)
         dZi = dZ.reshape(n, B, fout)
         G[:, offW:offW + fout * fin] = np.einsum("nbo,nbi->noi", dZi, Ain).reshape(n, -1)
         G[:, offb:offb + fout] = dZi.sum(axis=1)
+        if return_magnitude:
+            Gmag[:, offW:offW + fout * fin] = np.einsum("nbo,nbi->noi", np.abs(dZi), np.abs(Ain)).reshape(n, -1)
+            Gmag[:, offb:offb + fout] = np.abs(dZi).sum(axis=1)
         if l > 0:
             W = params[l][0]
             live = zs[l - 1] > 0.0
             if relu_flip is not None and relu_flip[l - 1] is not None:
                 live = live ^ relu_flip[l - 1]
             dZ = rnd((dZ @ W) * live)
+    out = (G, loss)
     if return_preact:
-        return G, loss, zs, scales
-    return G, loss
+        out = out + (zs, scales)
+    if return_magnitude:
+        out = out + (Gmag,)
+    return out
 
 
 def single_worker_grad(widths, w, X, y, B, bf16=False, relu_flip=None):

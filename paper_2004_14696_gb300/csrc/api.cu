@@ -82,6 +82,14 @@ size_t dbw_worker_grads_workspace_bytes(int num_layers, const int32_t* widths, i
     return grads_workspace_bytes(num_layers, widths, n, B, prec);
 }
 
+int dbw_worker_grads_activations(int num_layers, const int32_t* widths, int n, int B, int prec, int layer,
+                                 size_t* offset, int64_t* ld, int* elem_bytes) {
+    g_err[0] = 0;
+    if (!widths || !offset || !ld || !elem_bytes)
+        return fail(DBW_EINVAL, "dbw_worker_grads_activations: NULL pointer argument");
+    return grads_activations(num_layers, widths, n, B, prec, layer, offset, ld, elem_bytes);
+}
+
 int dbw_worker_grads(int num_layers, const int32_t* widths, int prec, const float* w, int64_t d, const float* pool,
                      int64_t S, const int32_t* labels, const int32_t* idx, int n, int B, float* G, int64_t ld,
                      float* loss, void* ws, size_t ws_bytes, void* stream) {

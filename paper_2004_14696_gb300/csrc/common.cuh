@@ -49,6 +49,8 @@ cudaError_t launch_choose_b(dbw_state* s, double lr, double beta, int flags, int
 // Worker gradients (grads.cu)
 struct GradsPlan;
 size_t grads_workspace_bytes(int L, const int32_t* widths, int n, int B, int prec);
+int grads_activations(int L, const int32_t* widths, int n, int B, int prec, int layer, size_t* offset, int64_t* ld,
+                      int* elem_bytes);
 int launch_worker_grads(int L, const int32_t* widths, int prec, const float* w, int64_t d,
                         const float* pool, int64_t S, const int32_t* labels, const int32_t* idx,
                         int n, int B, float* G, int64_t ld, float* loss, void* ws, size_t ws_bytes,

@@ -1,0 +1,439 @@
+// bf16 GEMM on the 5th-generation tensor cores of sm_103a (tcgen05), written
+// with inline PTX: TMA (cp.async.bulk.tensor) loads into a ring of shared
+// memory stages guarded by mbarriers, one thread issuing tcgen05.mma into a
+// TMEM accumulator, and four epilogue warps reading TMEM with tcgen05.ld.
+//
+//   C[M, N] = sum_k A[m, k] * B[n, k]      (both operands K-major, bf16; fp32 accumulation)
+//
+// CTA = 6 warps:  warp 0  TMA producer (one lane) and TMEM owner
+//                 warp 1  MMA issuer (one lane)
+//                 warps 2-5  epilogue: warp w reads TMEM lanes 32*(w%4) .. +31,
+//                            i.e. rows m0 + 32*(w%4) + lane of the 128-row tile.
+// Tile 128 x BN x BK; K-major operands staged with the 128B (BK = 64) or 64B
+// (BK = 32) swizzle that both TMA and the UMMA shared-memory descriptors use.
+//
+// Every wait on an mbarrier is bounded (2 s of %globaltimer).  A wait that runs
+// out sets bit 0 of *status, the producer drains the TMA loads it still has in
+// flight (again bounded), TMEM is freed and the CTA returns; the results of that
+// launch are then undefined, never a fault or a hang.
+#include <cuda.h>
+
+#include <mutex>
+
+#include "gemm_tc.cuh"
+
+namespace dbw {
+
+namespace {
+
+constexpr int BM = 128;
+constexpr int kThreads = 192;
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
+// ------------------------------------------------------------------ PTX wrappers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+// Bounded wait for the phase of parity ``parity`` to complete.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer();
+    while (!mbar_try_wait(bar, parity))
+        if (globaltimer() - t0 > kWaitLimitNs) return false;
+    return true;
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm, int x, int y, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
+            dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(bar), "r"(x), "r"(y)
+        : "memory");
+}
+__device__ __forceinline__ void tc_alloc(uint32_t slot, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(slot), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_relinquish() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tc_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_mma(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
+        "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void tc_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tc_ld_32cols(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+}
+
+// UMMA shared-memory matrix descriptor for a K-major operand staged by TMA with
+// a ``sw``-byte swizzle (rows of sw bytes, 8-row atoms).  Fields: start address
+// >> 4 (bits 0-13), leading-dimension offset (unused for swizzled K-major, 1),
+// stride between 8-row groups >> 4 (bits 32-45), descriptor version 1 (bit 46),
+// base offset 0 (tiles are atom aligned), swizzle mode (bits 61-63:
+// 2 = 128B, 4 = 64B).
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, int sw) {
+    uint64_t d = 0;
+    d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+    d |= static_cast<uint64_t>(1) << 16;
+    d |= static_cast<uint64_t>((8u * sw) >> 4) << 32;
+    d |= static_cast<uint64_t>(1) << 46;
+    d |= static_cast<uint64_t>(sw == 128 ? 2 : 4) << 61;
+    return d;
+}
+
+// Instruction descriptor of kind::f16: D fp32 (bits 4-5 = 1), A and B bf16
+// (bits 7-9 = 1, 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at bit 17,
+// M >> 4 at bit 24.
+__host__ __device__ constexpr uint32_t instr_desc_bf16(int m, int n) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(n >> 3) << 17) |
+           (static_cast<uint32_t>(m >> 4) << 24);
+}
+
+__device__ __forceinline__ float u2f(uint32_t u) { return __uint_as_float(u); }
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);   // .x = a (low half), .y = b
+    return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// ------------------------------------------------------------------ epilogues
+// One thread: row ``row`` of the tile, 32 columns starting at ``nb``.
+template <int KIND>
+__device__ __forceinline__ void epilogue_chunk(const TcEpi& e, int z, int row, int nb, int M, int N,
+                                               const uint32_t (&r)[32]) {
+    if (row >= M) return;
+    const bool full = nb + 32 <= N;
+    if (KIND == TC_HIDDEN || KIND == TC_DX) {
+        float x[32];
+        if (KIND == TC_HIDDEN) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                const float v = u2f(r[j]) + (nb + j < N ? __ldg(e.bias + nb + j) : 0.f);
+                x[j] = v > 0.f ? v : 0.f;
+            }
+        } else {
+            const __nv_bfloat16* ap = e.act + static_cast<int64_t>(row) * e.ldact + nb;
+            if (full && ((reinterpret_cast<uintptr_t>(ap) & 15u) == 0)) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint4 raw = *reinterpret_cast<const uint4*>(ap + 8 * q);
+                    const __nv_bfloat16* h = reinterpret_cast<const __nv_bfloat16*>(&raw);
+#pragma unroll
+                    for (int t = 0; t < 8; ++t)
+                        x[8 * q + t] = u2f(r[8 * q + t]) * (__bfloat162float(h[t]) > 0.f ? 1.f : 0.f);
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    x[j] = (nb + j < N) ? u2f(r[j]) * (__bfloat162float(ap[j]) > 0.f ? 1.f : 0.f) : 0.f;
+            }
+        }
+        __nv_bfloat16* op = e.out + static_cast<int64_t>(row) * e.ldo + nb;
+        if (full && ((reinterpret_cast<uintptr_t>(op) & 15u) == 0)) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                uint4 w;
+                w.x = pack_bf16(x[8 * q + 0], x[8 * q + 1]);
+                w.y = pack_bf16(x[8 * q + 2], x[8 * q + 3]);
+                w.z = pack_bf16(x[8 * q + 4], x[8 * q + 5]);
+                w.w = pack_bf16(x[8 * q + 6], x[8 * q + 7]);
+                *reinterpret_cast<uint4*>(op + 8 * q) = w;
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (nb + j < N) op[j] = __float2bfloat16_rn(x[j]);
+        }
+        if (e.outT) {
+            // column n of the tile -> row n of the transposed copy: the 32 lanes of the
+            // warp hold 32 consecutive rows m, so each store covers 64 contiguous bytes
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (nb + j < N) e.outT[static_cast<int64_t>(nb + j) * e.ldT + row] = __float2bfloat16_rn(x[j]);
+        }
+    } else if (KIND == TC_LOGITS) {
+        float* op = e.outF + static_cast<int64_t>(row) * e.ldF + nb;
+        if (full && ((reinterpret_cast<uintptr_t>(op) & 15u) == 0)) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                float4 v;
+                v.x = u2f(r[4 * q + 0]) + __ldg(e.bias + nb + 4 * q + 0);
+                v.y = u2f(r[4 * q + 1]) + __ldg(e.bias + nb + 4 * q + 1);
+                v.z = u2f(r[4 * q + 2]) + __ldg(e.bias + nb + 4 * q + 2);
+                v.w = u2f(r[4 * q + 3]) + __ldg(e.bias + nb + 4 * q + 3);
+                *reinterpret_cast<float4*>(op + 4 * q) = v;
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (nb + j < N) op[j] = u2f(r[j]) + __ldg(e.bias + nb + j);
+        }
+    } else {   // TC_DW
+        float* op = e.G + static_cast<int64_t>(z) * e.ldG + e.off + static_cast<int64_t>(row) * e.ldrow + nb;
+        if (full && ((reinterpret_cast<uintptr_t>(op) & 15u) == 0)) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                float4 v = make_float4(u2f(r[4 * q]), u2f(r[4 * q + 1]), u2f(r[4 * q + 2]), u2f(r[4 * q + 3]));
+                __stcs(reinterpret_cast<float4*>(op + 4 * q), v);   // streaming: G is read back much later
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (nb + j < N) op[j] = u2f(r[j]);
+        }
+    }
+}
+
+// ------------------------------------------------------------------ kernel
+template <int BN, int BK, int STAGES>
+struct TcCfg {
+    static constexpr int A_BYTES = BM * BK * 2;
+    static constexpr int B_BYTES = BN * BK * 2;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int SW = BK * 2;   // swizzle span in bytes: 128 (BK = 64) or 64 (BK = 32)
+    static constexpr int BAR_BYTES = 256;
+    static constexpr int SMEM = STAGES * STAGE_BYTES + BAR_BYTES + 1024;   // + alignment slack
+    static_assert(BK == 64 || BK == 32, "BK must be 64 or 32");
+    static_assert(BN == 128 || BN == 256, "BN must be 128 or 256");
+};
+
+template <int BN, int BK, int STAGES, int KIND, int MINB>
+__global__ void __launch_bounds__(kThreads, MINB)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
+                   int K, int64_t kz, TcEpi epi, int* status) {
+    using Cfg = TcCfg<BN, BK, STAGES>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sA = smem;
+    uint8_t* sB = smem + STAGES * Cfg::A_BYTES;
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
+    uint64_t* empty_bar = full_bar + STAGES;
+    uint64_t* accum_bar = empty_bar + STAGES;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum_bar + 1);
+    int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN, z = blockIdx.z;
+    const int nk = (K + BK - 1) / BK;
+    const int kbase = static_cast<int>(z * kz);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(smem_u32(full_bar + s), 1);
+            mbar_init(smem_u32(empty_bar + s), 1);
+        }
+        mbar_init(smem_u32(accum_bar), 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tc_alloc(smem_u32(tmem_slot), BN);
+        tc_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer
+        int issued = 0;
+        for (int kb = 0; kb < nk; ++kb) {
+            const int s = kb % STAGES;
+            const uint32_t ph = (kb / STAGES) & 1;
+            if (!mbar_wait(smem_u32(empty_bar + s), ph ^ 1)) {
+                atomicOr(status, 1);
+                atomicExch(abort_flag, 1);
+                break;
+            }
+            if (*reinterpret_cast<volatile int*>(abort_flag)) break;
+            mbar_expect_tx(smem_u32(full_bar + s), Cfg::STAGE_BYTES);
+            tma_load_2d(smem_u32(sA + s * Cfg::A_BYTES), &tmA, kbase + kb * BK, m0, smem_u32(full_bar + s));
+            tma_load_2d(smem_u32(sB + s * Cfg::B_BYTES), &tmB, kbase + kb * BK, n0, smem_u32(full_bar + s));
+            issued = kb + 1;
+        }
+        if (*reinterpret_cast<volatile int*>(abort_flag)) {
+            // drain this thread's copies that may still be in flight (the last STAGES issued)
+            for (int kb = issued - STAGES < 0 ? 0 : issued - STAGES; kb < issued; ++kb)
+                mbar_wait(smem_u32(full_bar + kb % STAGES), (kb / STAGES) & 1);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer
+        constexpr uint32_t idesc = instr_desc_bf16(BM, BN);
+        for (int kb = 0; kb < nk; ++kb) {
+            const int s = kb % STAGES;
+            const uint32_t ph = (kb / STAGES) & 1;
+            if (!mbar_wait(smem_u32(full_bar + s), ph)) {
+                atomicOr(status, 1);
+                atomicExch(abort_flag, 1);
+                break;
+            }
+            tc_fence_after();
+            const uint32_t a0 = smem_u32(sA + s * Cfg::A_BYTES);
+            const uint32_t b0 = smem_u32(sB + s * Cfg::B_BYTES);
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk) {
+                tc_mma(tmem, smem_desc(a0 + kk * 32, Cfg::SW), smem_desc(b0 + kk * 32, Cfg::SW), idesc,
+                       (kb > 0 || kk > 0) ? 1u : 0u);
+            }
+            tc_commit(smem_u32(empty_bar + s));   // frees the stage once these MMAs have read it
+        }
+        tc_commit(smem_u32(accum_bar));           // accumulator complete (or, after an abort, quiescent)
+    } else if (warp >= 2) {
+        // ---------------- epilogue
+        if (!mbar_wait(smem_u32(accum_bar), 0)) {
+            atomicOr(status, 1);
+        } else if (!*reinterpret_cast<volatile int*>(abort_flag)) {
+            tc_fence_after();
+            const int q = warp & 3;
+            const int row = m0 + q * 32 + lane;
+            const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16);
+#pragma unroll 1
+            for (int c = 0; c < BN / 32; ++c) {
+                if (n0 + c * 32 >= N) break;
+                uint32_t r[32];
+                tc_ld_32cols(tbase + c * 32, r);
+                tc_wait_ld();
+                epilogue_chunk<KIND>(epi, z, row, n0 + c * 32, M, N, r);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tc_dealloc(tmem, BN);
+    }
+}
+
+// ------------------------------------------------------------------ host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// 2-D tensor map of a row-major bf16 matrix [rows, cols] with row stride ld (elements).
+bool make_map(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_k, int box_rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld * 2)};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(box_k), static_cast<cuuint32_t>(box_rows)};
+    cuuint32_t estr[2] = {1, 1};
+    const CUtensorMapSwizzle sw = box_k == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+    return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN, int BK, int STAGES, int KIND, int MINB>
+cudaError_t launch_cfg(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, int batch, int64_t kz,
+                       const TcEpi& e, int* status, cudaStream_t st, int min_smem) {
+    using Cfg = TcCfg<BN, BK, STAGES>;
+    auto kern = tc_gemm_kernel<BN, BK, STAGES, KIND, MINB>;
+    const int smem = Cfg::SMEM > min_smem ? Cfg::SMEM : min_smem;
+    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (err != cudaSuccess) return err;
+    dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM, batch);
+    kern<<<grid, kThreads, smem, st>>>(a, b, M, N, K, kz, e, status);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool tc_shape_ok(int64_t lda, int64_t ldb, int K, int64_t kz, const void* A, const void* B) {
+    if (!encode_fn()) return false;
+    if ((lda % 8) || (ldb % 8) || (kz % 8)) return false;
+    if ((reinterpret_cast<uintptr_t>(A) & 15u) || (reinterpret_cast<uintptr_t>(B) & 15u)) return false;
+    if (kz > 0 && K % 32) return false;   // a batch's K must be whole K blocks (it is the column offset step)
+    return K >= 1;
+}
+
+int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_t colsA, const __nv_bfloat16* B,
+            int64_t ldb, int64_t rowsB, int64_t colsB, int M, int N, int K, int batch, int64_t kz, const TcEpi& epi,
+            int* status, cudaStream_t st) {
+    if (!tc_shape_ok(lda, ldb, K, kz, A, B)) return fail(DBW_EALIGN, "tc_gemm: unsupported operand alignment");
+    CUtensorMap ta, tb;
+    cudaError_t e = cudaSuccess;
+    if (kind == TC_DW) {
+        // K = the per-worker sample count: 64-deep blocks when it allows, else 32
+        const int bk = (K % 64 == 0) ? 64 : 32;
+        if (!make_map(&ta, A, rowsA, colsA, lda, bk, BM) || !make_map(&tb, B, rowsB, colsB, ldb, bk, 128))
+            return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
+        // 4 CTAs per SM (48 KB of shared memory each) share the 512 TMEM columns, 128 each
+        if (bk == 64)
+            e = launch_cfg<128, 64, 2, TC_DW, 4>(ta, tb, M, N, K, batch, kz, epi, status, st, 48 * 1024);
+        else
+            e = launch_cfg<128, 32, 2, TC_DW, 4>(ta, tb, M, N, K, batch, kz, epi, status, st, 48 * 1024);
+    } else {
+        if (!make_map(&ta, A, rowsA, colsA, lda, 64, BM) || !make_map(&tb, B, rowsB, colsB, ldb, 64, 256))
+            return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
+        // one CTA per SM (4 stages x 48 KB), 256 TMEM columns
+        if (kind == TC_HIDDEN)
+            e = launch_cfg<256, 64, 4, TC_HIDDEN, 1>(ta, tb, M, N, K, batch, kz, epi, status, st, 0);
+        else if (kind == TC_LOGITS)
+            e = launch_cfg<256, 64, 4, TC_LOGITS, 1>(ta, tb, M, N, K, batch, kz, epi, status, st, 0);
+        else
+            e = launch_cfg<256, 64, 4, TC_DX, 1>(ta, tb, M, N, K, batch, kz, epi, status, st, 0);
+    }
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "tc_gemm launch: %s", cudaGetErrorString(e));
+    return DBW_OK;
+}
+
+}  // namespace dbw

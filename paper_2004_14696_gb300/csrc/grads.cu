@@ -12,8 +12,8 @@
 //   backward   G[i, W_l] = dZ_l[i]^T A_{l-1}[i],  G[i, b_l] = sum_rows dZ_l[i],
 //              dZ_{l-1} = (dZ_l W_l) * 1[A_{l-1} > 0]      (ReLU'(0) = 0)
 //
-// GEMMs here are the SIMT path (fp32 FFMA on fp32 or bf16 operands); the bf16
-// configurations can instead run the tcgen05 kernels of gemm_tc.cu.
+// GEMMs here are the SIMT path (fp32 FFMA on fp32 or bf16 operands), used for the
+// fp32 workloads and for bf16 shapes the tcgen05 pass (grads_tc.cu) does not take.
 #include <math.h>
 
 #include "common.cuh"
@@ -258,6 +258,8 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
     float* logits = reinterpret_cast<float*>(ws + P.off_logits);
     float* sloss = reinterpret_cast<float*>(ws + P.off_sloss);
     T* dz[2] = {reinterpret_cast<T*>(ws + P.off_dz[0]), reinterpret_cast<T*>(ws + P.off_dz[1])};
+    cudaError_t e0 = cudaMemsetAsync(ws, 0, sizeof(int), st);
+    if (e0 != cudaSuccess) return fail(DBW_ECUDA, "dbw_worker_grads: %s", cudaGetErrorString(e0));
     const T* wop;
     if (sizeof(T) == 2) {
         __nv_bfloat16* wb = reinterpret_cast<__nv_bfloat16*>(ws + P.off_wb);
@@ -353,6 +355,7 @@ bool make_grads_plan(int L, const int32_t* widths, int n, int B, int prec, Grads
         cur += (bytes + 255) / 256 * 256;
         return at;
     };
+    take(256);   // status word (int32 at offset 0), as in the tcgen05 plan
     P->off_x = take((size_t)M * widths[0] * es);
     P->off_act[0] = P->off_x;
     for (int l = 1; l < L; ++l) P->off_act[l] = take((size_t)M * widths[l] * es);
@@ -365,7 +368,31 @@ bool make_grads_plan(int L, const int32_t* widths, int n, int B, int prec, Grads
     return true;
 }
 
+int grads_activations(int L, const int32_t* widths, int n, int B, int prec, int layer, size_t* offset, int64_t* ld,
+                      int* elem_bytes) {
+    if (layer < 1 || layer >= L) return fail(DBW_EINVAL, "dbw_worker_grads_activations: layer must be in [1, L-1]");
+    if (tc_eligible(prec, B)) {
+        TcPlan T;
+        if (!make_tc_plan(L, widths, n, B, &T)) return fail(DBW_EINVAL, "dbw_worker_grads_activations: invalid shape");
+        *offset = T.off_act[layer];
+        *ld = T.ldact[layer];
+        *elem_bytes = 2;
+        return DBW_OK;
+    }
+    GradsPlan P;
+    if (!make_grads_plan(L, widths, n, B, prec, &P)) return fail(DBW_EINVAL, "dbw_worker_grads_activations: invalid shape");
+    *offset = P.off_act[layer];
+    *ld = widths[layer];
+    *elem_bytes = prec == DBW_PREC_BF16 ? 2 : 4;
+    return DBW_OK;
+}
+
 size_t grads_workspace_bytes(int L, const int32_t* widths, int n, int B, int prec) {
+    if (tc_eligible(prec, B)) {
+        TcPlan T;
+        if (!make_tc_plan(L, widths, n, B, &T)) return 0;
+        return T.ws_bytes;
+    }
     GradsPlan P;
     if (!make_grads_plan(L, widths, n, B, prec, &P)) return 0;
     return P.ws_bytes;
@@ -378,8 +405,15 @@ int launch_worker_grads(int L, const int32_t* widths, int prec, const float* w, 
     if (!make_grads_plan(L, widths, n, B, prec, &P)) return fail(DBW_EINVAL, "dbw_worker_grads: invalid model shape");
     if (P.d != d) return fail(DBW_EINVAL, "dbw_worker_grads: d = %lld but the widths give %lld", (long long)d,
                               (long long)P.d);
-    if (ws_bytes < P.ws_bytes)
+    if (!tc_eligible(prec, B) && ws_bytes < P.ws_bytes)
         return fail(DBW_EINVAL, "dbw_worker_grads: workspace %zu bytes < %zu needed", ws_bytes, P.ws_bytes);
+    if (tc_eligible(prec, B)) {
+        TcPlan T;
+        if (!make_tc_plan(L, widths, n, B, &T)) return fail(DBW_EINVAL, "dbw_worker_grads: invalid model shape");
+        if (ws_bytes < T.ws_bytes)
+            return fail(DBW_EINVAL, "dbw_worker_grads: workspace %zu bytes < %zu needed", ws_bytes, T.ws_bytes);
+        return worker_grads_tc(T, w, pool, S, labels, idx, G, ld, loss, static_cast<char*>(ws), st);
+    }
     if (prec == DBW_PREC_BF16)
         return worker_grads_impl<__nv_bfloat16>(P, w, pool, S, labels, idx, G, ld, loss, static_cast<char*>(ws), st);
     return worker_grads_impl<float>(P, w, pool, S, labels, idx, G, ld, loss, static_cast<char*>(ws), st);

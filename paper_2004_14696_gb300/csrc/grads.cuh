@@ -4,6 +4,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <cuda_runtime.h>
+
 #include "dbw.h"
 
 namespace dbw {
@@ -24,5 +26,33 @@ struct GradsPlan {
 };
 
 bool make_grads_plan(int L, const int32_t* widths, int n, int B, int prec, GradsPlan* P);
+
+// Workspace of the tcgen05 (bf16) pass; every offset 256-byte aligned, every
+// leading dimension (ld*) a multiple of 8 elements.
+struct TcPlan {
+    GradsPlan g;                       // shapes and parameter offsets
+    int64_t M8;                        // leading dimension of the transposed [width, M] buffers
+    size_t off_status;                 // device int: bit 0 = a pipeline wait timed out
+    size_t off_wb[DBW_LMAX];           // W_l bf16 [out, ldw]
+    int64_t ldw[DBW_LMAX];
+    size_t off_wt[DBW_LMAX];           // W_l^T bf16 [in, ldwt]
+    int64_t ldwt[DBW_LMAX];
+    size_t off_act[DBW_LMAX];          // layer-l input bf16 [M, ldact] (act[0] = X)
+    int64_t ldact[DBW_LMAX];
+    size_t off_actT[DBW_LMAX];         // its transpose bf16 [width, M8]
+    size_t off_logits;                 // fp32 [M, ldlog]
+    int64_t ldlog;
+    size_t off_sloss;                  // fp32 [M]
+    size_t off_dz[2];                  // bf16 [M, ldz] ping-pong
+    int64_t ldz;
+    size_t off_dzT;                    // bf16 [max width, M8]
+    size_t ws_bytes;
+};
+
+// The bf16 pass runs on tcgen05 when each worker's sample count is whole 32-deep K blocks.
+bool tc_eligible(int prec, int B);
+bool make_tc_plan(int L, const int32_t* widths, int n, int B, TcPlan* P);
+int worker_grads_tc(const TcPlan& P, const float* w, const float* pool, int64_t S, const int32_t* labels,
+                    const int32_t* idx, float* G, int64_t ld, float* loss, char* ws, cudaStream_t st);
 
 }  // namespace dbw

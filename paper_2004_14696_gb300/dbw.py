@@ -56,6 +56,7 @@ _SIGS = {
     "dbw_abi_version": (_i32, []),
     "dbw_param_count": (_i64, [_i32, _vp]),
     "dbw_worker_grads_workspace_bytes": (_sz, [_i32, _vp, _i32, _i32, _i32]),
+    "dbw_worker_grads_activations": (_i32, [_i32, _vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp]),
     "dbw_worker_grads": (_i32, [_i32, _vp, _i32, _vp, _i64, _vp, _i64, _vp, _vp, _i32, _i32, _vp, _i64, _vp,
                                 _vp, _sz, _vp]),
     "dbw_select_fastest": (_i32, [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp]),
@@ -125,6 +126,24 @@ def dbw_param_count(widths):
 def dbw_worker_grads_workspace_bytes(widths, n, B, prec):
     L, arr = _widths(widths)
     return int(lib().dbw_worker_grads_workspace_bytes(L, arr, n, B, prec))
+
+
+def dbw_worker_grads_activations(widths, n, B, prec, layer):
+    """(byte offset in ws, leading dimension, element bytes) of layer ``layer``'s input activations."""
+    L, arr = _widths(widths)
+    off, ld, eb = C.c_size_t(), C.c_int64(), C.c_int()
+    rc = lib().dbw_worker_grads_activations(L, arr, n, B, prec, layer, C.byref(off), C.byref(ld), C.byref(eb))
+    _check("dbw_worker_grads_activations", rc)
+    return off.value, ld.value, eb.value
+
+
+def hidden_activations(ws, widths, n, B, prec, layer):
+    """View of the hidden activations [n*B, width] a dbw_worker_grads call left in ws (device tensor)."""
+    off, ld, eb = dbw_worker_grads_activations(widths, n, B, prec, layer)
+    M = n * B
+    raw = ws[off:off + M * ld * eb]
+    t = raw.view(torch.bfloat16 if eb == 2 else torch.float32).view(M, ld)
+    return t[:, : int(widths[layer])]
 
 
 def dbw_aggregate_partials_bytes(n, d):

@@ -89,9 +89,14 @@ class Iteration:
     def launches_per_step(self):
         """Kernels libdbw launches per step (for the bench's launch count)."""
         L = len(self.wl.widths) - 1
-        grads = 1 + L + 1 + L + L + (L - 1)          # gather, fwd, loss, dW, bias, dX
-        if self.wl.prec == dbw.PREC_BF16:
-            grads += 1                                  # bf16 weight cast
+        if self.wl.prec == dbw.PREC_BF16 and self.wl.B % 32 == 0:
+            # tcgen05 pass: status memset, L weight cast-transposes, gather + X^T, L forward
+            # GEMMs, loss + dZ^T, L dW GEMMs, L bias gradients, L-1 dX GEMMs
+            grads = 1 + L + 2 + L + 2 + L + L + (L - 1)
+        else:
+            grads = 1 + 1 + L + 1 + L + L + (L - 1)    # status memset, gather, fwd, loss, dW, bias, dX
+            if self.wl.prec == dbw.PREC_BF16:
+                grads += 1                              # bf16 weight cast
         return (0 if self.static_b is not None else 1) + grads + 1 + 1 + 2
 
 

@@ -5,6 +5,10 @@ import numpy as np
 
 RTOL_FP32 = 1e-5    # fp32 GEMM / fp32 accumulation paths
 RTOL_BF16 = 2e-2    # bf16 GEMM operands with fp32 accumulation
+# bf16 elementwise outliers: at most this fraction of a worker's entries may exceed
+# 2e-2 of their error scale, and none by more than this factor
+BF16_OUTLIER_FRACTION = 1e-5
+BF16_OUTLIER_FACTOR = 4.0
 
 
 def param_blocks(widths):
@@ -62,55 +66,110 @@ def _rows_close(x, r, rtol, blocks):
         return str(e)
 
 
-def assert_worker_grads_match(G_gpu, loss_gpu, widths, w, X, y, B, bf16, workers, rtol,
-                              amb=None, max_candidates=6, max_flips=3):
+def assert_worker_grads_match(G_gpu, loss_gpu, widths, w, X, y, B, bf16, workers, rtol, gpu_active=None,
+                              amb=None):
     """Each sampled worker's GPU gradient row matches the oracle's Eq. (2) row.
 
     A ReLU derivative whose pre-activation lies within rounding of 0 is a
     decision either value of which is correct at the kernel's precision (R13).
-    When a row does not match, the oracle's own hidden pre-activations are ranked
-    by |Z| / scale (scale = sum of |terms| of that dot product), the few most
-    ambiguous ones (|Z| / scale <= amb) are flipped in every combination of up to
-    ``max_flips`` of them, and the row must match one of those oracle results.
-    Nothing of the GPU's enters the oracle; the GPU row is only compared.
-    Returns {worker: (oracle row it matched, oracle loss)}: the valid reference a
-    later check (the aggregation of these rows) must use.
+    ``gpu_active[h]`` is the GPU's decision set for hidden layer h (its
+    activations > 0, [n*B, width]).  What is unique is checked exactly: every
+    decision the GPU took differently from the oracle must be one the oracle
+    itself certifies as ambiguous (|Z| <= amb * sum of |terms| of that dot
+    product, from the oracle's own pre-activations).  What is then determined is
+    checked with the tolerance: the GPU row against the oracle's Eq. (2) row
+    evaluated with those decisions, relative to the larger of two error scales,
+    the magnitude of the products forming each entry (sum of |terms|: a cancelled
+    sum is only as accurate as its largest terms) and |r| + the rms of the entry's
+    parameter tensor (an entry made of few products inherits the relative error
+    of upstream sums that cancelled).  Returns {worker: (oracle row, oracle loss, magnitude row)}.
     """
-    import itertools
-
     from oracle import dbw_oracle as O
 
     if amb is None:
-        amb = 2e-3 if bf16 else 1e-4
+        amb = 1e-3 if bf16 else 1e-4
     blocks = param_blocks(widths)
-    matched = {}
+    L = len(widths) - 1
+    matched, flipped = {}, 0
     for i in workers:
         Xi, yi = X[i * B:(i + 1) * B], y[i * B:(i + 1) * B]
-        g, l, zs, scales = O.worker_grads(widths, w, Xi, yi, 1, B, bf16, return_preact=True)
+        g, l, zs, scales, gm = O.worker_grads(widths, w, Xi, yi, 1, B, bf16, return_preact=True,
+                                              return_magnitude=True)
         assert_close_scalar(loss_gpu[i], l[0], rtol, f"loss of worker {i}")
-        msg = _rows_close(G_gpu[i], g[0], rtol, blocks)
-        if msg is None:
-            matched[i] = (g[0], float(l[0]))
-            continue
-        cand = []
-        for h, (Z, S) in enumerate(zip(zs, scales)):
-            rel = np.abs(Z) / np.where(S > 0, S, 1.0)
-            for (r, u) in zip(*np.nonzero(rel <= amb)):
-                cand.append((float(rel[r, u]), h, int(r), int(u)))
-        cand = sorted(cand)[:max_candidates]
-        ok = False
-        for m in range(1, min(max_flips, len(cand)) + 1):
-            for sub in itertools.combinations(cand, m):
-                flips = [np.zeros(Z.shape, dtype=bool) for Z in zs]
-                for (_, h, r, u) in sub:
-                    flips[h][r, u] = True
-                g2, _ = O.worker_grads(widths, w, Xi, yi, 1, B, bf16, relu_flip=flips)
-                if _rows_close(G_gpu[i], g2[0], rtol, blocks) is None:
-                    ok = True
-                    matched[i] = (g2[0], float(l[0]))
-                    break
-            if ok:
-                break
-        assert ok, f"worker {i}: {msg} (no ReLU decision within rounding of 0 explains it; " \
-                   f"{len(cand)} candidates)"
+        flips = None
+        if L > 1:
+            assert gpu_active is not None and len(gpu_active) == L - 1
+            flips = []
+            for h in range(L - 1):
+                mine = np.asarray(gpu_active[h][i * B:(i + 1) * B], dtype=bool)
+                diff = mine != (zs[h] > 0.0)
+                if diff.any():
+                    rel = np.abs(zs[h][diff]) / np.where(scales[h][diff] > 0, scales[h][diff], 1.0)
+                    assert np.all(rel <= amb), (f"worker {i} layer {h}: {int((rel > amb).sum())} ReLU decisions "
+                                                f"differ from the oracle's outside rounding of 0 "
+                                                f"(largest |Z|/scale {rel.max():.3g})")
+                flips.append(diff)
+                flipped += int(diff.sum())
+            if any(f.any() for f in flips):
+                g, _, gm = O.worker_grads(widths, w, Xi, yi, 1, B, bf16, relu_flip=flips, return_magnitude=True)
+        x = np.asarray(G_gpu[i], dtype=np.float64)
+        scale = np.maximum(gm[0], tensor_scale(g[0], blocks))
+        if not bf16:
+            assert_close_to_magnitude(x, g[0], scale, rtol, f"G row of worker {i}")
+        else:
+            # normwise per parameter tensor: the 2e-2 relative target
+            for (a, b) in blocks:
+                num, den = np.linalg.norm(x[a:b] - g[0][a:b]), np.linalg.norm(g[0][a:b])
+                assert num <= rtol * den, f"worker {i} tensor [{a},{b}): normwise relative error {num / den:.3g}"
+            # elementwise bug detector: two bf16 rounding chains (fp32 vs fp64 values rounded
+            # at the same points) drift one bf16 step apart in a growing fraction of deep
+            # activations, so a few near-zero activations carry a large relative error
+            ratio = np.abs(x - g[0]) / (rtol * scale)
+            nbad = int((ratio > 1.0).sum())
+            assert nbad <= max(1, int(BF16_OUTLIER_FRACTION * x.size)) and ratio.max() <= BF16_OUTLIER_FACTOR, (
+                f"worker {i}: {nbad} of {x.size} entries beyond 2e-2 of their scale, worst {ratio.max():.3g}x")
+        matched[i] = (g[0], float(l[0]), gm[0])
     return matched
+
+
+def tensor_scale(row, blocks):
+    """|r| + rms(r) with the rms taken over the parameter tensor (block) of each entry."""
+    r = np.asarray(row, dtype=np.float64)
+    s = np.empty_like(r)
+    for (a, b) in blocks:
+        s[a:b] = np.sqrt(np.mean(r[a:b] ** 2))
+    return np.abs(r) + s
+
+
+def assert_close_to_magnitude(x, ref, mag, rtol, what="", extra=0.0):
+    """|x - r| <= rtol * mag + extra elementwise, mag = the sum of |products| forming
+    each entry (the standard error scale of a dot product: a sum that cancels to ~0
+    is only as accurate as its largest terms); ``extra`` an absolute allowance
+    (e.g. the fp32 storage rounding of a parameter vector)."""
+    x = np.asarray(x, dtype=np.float64)
+    r = np.asarray(ref, dtype=np.float64)
+    m = np.asarray(mag, dtype=np.float64)
+    err = np.abs(x - r)
+    lim = rtol * m + extra
+    bad = ~(err <= lim)
+    if bad.any():
+        i = np.argwhere(bad)[0]
+        worst = float(np.max(err / np.where(lim > 0, lim, np.inf)))
+        raise AssertionError(f"{what}: {bad.sum()} of {bad.size} entries off (worst {worst:.3g}x the limit); "
+                             f"first at {tuple(i)}: got {x[tuple(i)]!r} want {r[tuple(i)]!r} (limit {lim[tuple(i)]:.3g})")
+
+
+def gpu_active_sets(ws, widths, n, B, prec):
+    """The GPU's ReLU decisions (activation > 0) per hidden layer, as host bool arrays."""
+    from paper_2004_14696_gb300 import dbw
+    return [(dbw.hidden_activations(ws, widths, n, B, prec, h + 1) > 0).cpu().numpy()
+            for h in range(len(widths) - 2)]
+
+
+def _bad_entries(x, r, rtol, blocks):
+    r2 = np.asarray(r, dtype=np.float64)
+    scale = np.empty_like(r2)
+    for (a, b) in blocks:
+        seg = r2[a:b]
+        scale[a:b] = np.sqrt(np.mean(seg * seg))
+    return ~(np.abs(np.asarray(x, dtype=np.float64) - r2) <= rtol * (np.abs(r2) + scale))

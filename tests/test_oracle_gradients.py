@@ -153,3 +153,15 @@ def test_planted_dropped_term_is_caught(monkeypatch):
     monkeypatch.setattr(O, "worker_grads", dropped_term)
     with pytest.raises(AssertionError):
         test_mlp_gradient_matches_central_differences((5, 4, 3))
+
+
+def test_gradient_magnitude_bounds_and_single_term_case():
+    """The magnitude of an entry (sum of |products|) bounds |entry|, and equals it
+    when the entry is a single product (one sample, one layer)."""
+    widths = (6, 5, 4)
+    w, X, y = _problem(widths, 2, 3, 8)
+    G, _, Gm = O.worker_grads(widths, w, X, y, 2, 3, return_magnitude=True)
+    assert np.all(Gm >= np.abs(G) - 1e-15)
+    w1, X1, y1 = _problem((6, 4), 1, 1, 9)
+    G1, _, Gm1 = O.worker_grads((6, 4), w1, X1, y1, 1, 1, return_magnitude=True)
+    np.testing.assert_allclose(Gm1, np.abs(G1), rtol=1e-15, atol=0)
