@@ -152,6 +152,7 @@ def run_dbw(args, rank, world, local_rank):
         from dataclasses import replace
         wl = replace(wl, seed_offset=wl.seed_offset + 1000 * rank)
     it = Iteration(wl, device=dev)
+    w_init = it.w.clone()
     n, B = wl.n, wl.B
     total = W + K
     idx_h = np.stack([inputs.minibatch_indices(wl.seed, t, n, B, wl.S) for t in range(total)])
@@ -214,7 +215,10 @@ def run_dbw(args, rank, world, local_rank):
     # the same steps through the public API with host buffers: per step, pinned
     # host -> device copies of the minibatch indices and times, the iteration,
     # and a device -> host read of the step's statistics (loss, k, V, ...).
+    # the e2e leg replays the very same iterations: parameters and estimator state restart
     it2 = it
+    it2.w.copy_(w_init)
+    dbw.dbw_state_init(it2.state, n, wl.D, stream)
     idx_pin = torch.from_numpy(idx_h).pin_memory()
     tim_pin = torch.from_numpy(tim_h).pin_memory()
     stats_pin = torch.empty(dbw.STATS_LEN, dtype=torch.float64).pin_memory()

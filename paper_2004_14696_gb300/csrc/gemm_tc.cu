@@ -134,6 +134,28 @@ __host__ __device__ constexpr uint32_t instr_desc_bf16(int m, int n) {
 
 __device__ __forceinline__ float u2f(uint32_t u) { return __uint_as_float(u); }
 
+// TMA bulk tensor store (shared -> global) of a 3-D box, and its bulk-group bookkeeping.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* tm, uint32_t src, int x, int y, int z) {
+    asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+                     reinterpret_cast<uint64_t>(tm)),
+                 "r"(src), "r"(x), "r"(y), "r"(z)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// wait until at most N committed bulk groups of this thread still read shared memory
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// make this thread's generic-proxy shared-memory writes visible to the async proxy (TMA)
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
     const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);   // .x = a (low half), .y = b
     return *reinterpret_cast<const uint32_t*>(&h);
@@ -349,6 +371,199 @@ __global__ void __launch_bounds__(kThreads, MINB)
     }
 }
 
+// ------------------------------------------------------------------ persistent dW kernel
+// Per-worker weight gradient G[z, off + m*ldrow + n] = sum_{k < K} A[m, z*K + k] B[n, z*K + k]
+// (A = dZ^T [out, M], B = A_{l-1}^T [in, M], K = B samples), written by TMA bulk
+// stores.  The kernel is bound by writing G (K is small), so it is built around
+// the store: a persistent grid (one CTA per SM) walks the tiles (worker-major),
+// the MMA of tile i+1 runs into the second of two 256-column TMEM accumulators
+// while the epilogue drains tile i, and each epilogue warp moves its 32 x 32 fp32
+// chunks TMEM -> registers -> 128B-swizzled shared memory (conflict-free) -> one
+// TMA store, double-buffered.
+constexpr int DW_BN = 256;
+constexpr int DW_CHUNK_BYTES = 32 * 32 * 4;   // one warp's 32 rows x 32 fp32 columns
+
+template <int BK, int STAGES>
+struct DwCfg {
+    static constexpr int A_BYTES = BM * BK * 2;
+    static constexpr int B_BYTES = DW_BN * BK * 2;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int SW = BK * 2;
+    static constexpr int STAGING = 4 * 2 * DW_CHUNK_BYTES;   // 4 epilogue warps x 2 buffers
+    static constexpr int BAR_BYTES = 256;
+    static constexpr int SMEM = STAGES * STAGE_BYTES + STAGING + BAR_BYTES + 1024;
+};
+
+template <int BK, int STAGES>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                 const __grid_constant__ CUtensorMap tmG, int Mr, int Nr, int K, int batch, int* status) {
+    using Cfg = DwCfg<BK, STAGES>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sA = smem;
+    uint8_t* sB = smem + STAGES * Cfg::A_BYTES;
+    uint8_t* stage_out = smem + STAGES * Cfg::STAGE_BYTES;   // 1024-aligned (stage sizes are)
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(stage_out + Cfg::STAGING);
+    uint64_t* empty_bar = full_bar + STAGES;
+    uint64_t* tfull_bar = empty_bar + STAGES;    // [2] accumulator ready
+    uint64_t* tempty_bar = tfull_bar + 2;        // [2] accumulator drained (4 epilogue warps)
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty_bar + 2);
+    int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int mt_n = (Mr + BM - 1) / BM, nt_n = (Nr + DW_BN - 1) / DW_BN;
+    const int tiles_per_z = mt_n * nt_n;
+    const long long total = static_cast<long long>(tiles_per_z) * batch;
+    const int nk = (K + BK - 1) / BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(smem_u32(full_bar + s), 1);
+            mbar_init(smem_u32(empty_bar + s), 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(smem_u32(tfull_bar + a), 1);
+            mbar_init(smem_u32(tempty_bar + a), 4);
+        }
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tc_alloc(smem_u32(tmem_slot), 2 * DW_BN);
+        tc_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    volatile int* vabort = abort_flag;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer: every k block of every tile this CTA owns
+        long long g = 0;
+        long long issued = 0;
+        for (long long t = blockIdx.x; t < total && !*vabort; t += gridDim.x) {
+            const int z = static_cast<int>(t / tiles_per_z);
+            const int rem = static_cast<int>(t % tiles_per_z);
+            const int m0 = (rem / nt_n) * BM, n0 = (rem % nt_n) * DW_BN;
+            for (int kb = 0; kb < nk; ++kb, ++g) {
+                const int s = static_cast<int>(g % STAGES);
+                const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
+                if (!mbar_wait(smem_u32(empty_bar + s), ph ^ 1)) {
+                    atomicOr(status, 1);
+                    *vabort = 1;
+                    break;
+                }
+                mbar_expect_tx(smem_u32(full_bar + s), Cfg::STAGE_BYTES);
+                const int kx = z * K + kb * BK;
+                tma_load_2d(smem_u32(sA + s * Cfg::A_BYTES), &tmA, kx, m0, smem_u32(full_bar + s));
+                tma_load_2d(smem_u32(sB + s * Cfg::B_BYTES), &tmB, kx, n0, smem_u32(full_bar + s));
+                issued = g + 1;
+            }
+        }
+        if (*vabort) {
+            for (long long q = issued - STAGES < 0 ? 0 : issued - STAGES; q < issued; ++q)
+                mbar_wait(smem_u32(full_bar + q % STAGES), static_cast<uint32_t>((q / STAGES) & 1));
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer
+        constexpr uint32_t idesc = instr_desc_bf16(BM, DW_BN);
+        long long g = 0;
+        int i = 0;
+        for (long long t = blockIdx.x; t < total && !*vabort; t += gridDim.x, ++i) {
+            const int acc = i & 1;
+            const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
+            if (!mbar_wait(smem_u32(tempty_bar + acc), aph ^ 1)) {
+                atomicOr(status, 1);
+                *vabort = 1;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t dcol = tmem + static_cast<uint32_t>(acc * DW_BN);
+            bool ok = true;
+            for (int kb = 0; kb < nk; ++kb, ++g) {
+                const int s = static_cast<int>(g % STAGES);
+                const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
+                if (!mbar_wait(smem_u32(full_bar + s), ph)) {
+                    atomicOr(status, 1);
+                    *vabort = 1;
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t a0 = smem_u32(sA + s * Cfg::A_BYTES);
+                const uint32_t b0 = smem_u32(sB + s * Cfg::B_BYTES);
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk)
+                    tc_mma(dcol, smem_desc(a0 + kk * 32, Cfg::SW), smem_desc(b0 + kk * 32, Cfg::SW), idesc,
+                           (kb > 0 || kk > 0) ? 1u : 0u);
+                tc_commit(smem_u32(empty_bar + s));
+            }
+            tc_commit(smem_u32(tfull_bar + acc));
+            if (!ok) break;
+        }
+    } else if (warp >= 2) {
+        // ---------------- epilogue: TMEM -> registers -> swizzled smem -> TMA store
+        const int q = warp & 3;
+        uint8_t* mybuf = stage_out + q * 2 * DW_CHUNK_BYTES;
+        int nbuf = 0;
+        int i = 0;
+        for (long long t = blockIdx.x; t < total; t += gridDim.x, ++i) {
+            const int acc = i & 1;
+            const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
+            if (!mbar_wait(smem_u32(tfull_bar + acc), aph)) {
+                atomicOr(status, 1);
+                *vabort = 1;
+                break;
+            }
+            if (*vabort) break;
+            tc_fence_after();
+            const int z = static_cast<int>(t / tiles_per_z);
+            const int rem = static_cast<int>(t % tiles_per_z);
+            const int m0 = (rem / nt_n) * BM, n0 = (rem % nt_n) * DW_BN;
+            const uint32_t tbase = tmem + static_cast<uint32_t>(acc * DW_BN) + (static_cast<uint32_t>(q * 32) << 16);
+            const int row0 = m0 + q * 32;
+#pragma unroll 1
+            for (int c = 0; c < DW_BN / 32; ++c) {
+                const int col0 = n0 + c * 32;
+                if (col0 >= Nr || row0 >= Mr) break;   // whole chunk outside the tensor (warp-uniform)
+                uint32_t r[32];
+                tc_ld_32cols(tbase + c * 32, r);
+                tc_wait_ld();
+                // this buffer was last handed to a TMA store two chunks ago: wait until read
+                if (lane == 0) bulk_wait_read<1>();
+                __syncwarp();
+                uint8_t* buf = mybuf + nbuf * DW_CHUNK_BYTES;
+                // row ``lane``: 8 chunks of 16 bytes, chunk j at (j ^ (lane & 7)) * 16 (128B swizzle)
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    uint4 v = make_uint4(r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
+                    *reinterpret_cast<uint4*>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) = v;
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_3d(&tmG, smem_u32(buf), col0, row0, z);
+                    bulk_commit();
+                }
+                nbuf ^= 1;
+            }
+            // every tcgen05.ld of this accumulator has completed (wait::ld above)
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(tempty_bar + acc));
+        }
+        if (lane == 0) bulk_wait_all();
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tc_dealloc(tmem, 2 * DW_BN);
+    }
+}
+
 // ------------------------------------------------------------------ host side
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -380,6 +595,34 @@ bool make_map(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int
     return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
               CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// 3-D tensor map over the fp32 weight-gradient block of every worker:
+// element (n, m, z) at base + z*ldG + m*ldrow + n, box 32 x 32 x 1, 128B swizzle.
+bool make_g_map(CUtensorMap* tm, const float* base, int64_t Nr, int64_t Mr, int64_t batch, int64_t ldrow,
+                int64_t ldG) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(Nr), static_cast<cuuint64_t>(Mr), static_cast<cuuint64_t>(batch)};
+    cuuint64_t strides[2] = {static_cast<cuuint64_t>(ldrow * 4), static_cast<cuuint64_t>(ldG * 4)};
+    cuuint32_t box[3] = {32, 32, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return fn(tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BK, int STAGES>
+cudaError_t launch_dw(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& g, int Mr, int Nr, int K,
+                      int batch, int* status, cudaStream_t st) {
+    using Cfg = DwCfg<BK, STAGES>;
+    auto kern = tc_dw_kernel<BK, STAGES>;
+    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    if (err != cudaSuccess) return err;
+    const long long tiles = static_cast<long long>((Mr + BM - 1) / BM) * ((Nr + DW_BN - 1) / DW_BN) * batch;
+    const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
+    kern<<<grid, kThreads, Cfg::SMEM, st>>>(a, b, g, Mr, Nr, K, batch, status);
+    return cudaGetLastError();
 }
 
 template <int BN, int BK, int STAGES, int KIND, int MINB>
@@ -414,6 +657,18 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
     if (kind == TC_DW) {
         // K = the per-worker sample count: 64-deep blocks when it allows, else 32
         const int bk = (K % 64 == 0) ? 64 : 32;
+        const float* gbase = epi.G + epi.off;
+        const bool store_ok = ((reinterpret_cast<uintptr_t>(gbase) & 15u) == 0) && (epi.ldrow % 4 == 0) &&
+                              (epi.ldG % 4 == 0) && M >= 1 && N >= 1;
+        CUtensorMap tg;
+        if (store_ok && make_map(&ta, A, rowsA, colsA, lda, bk, BM) &&
+            make_map(&tb, B, rowsB, colsB, ldb, bk, DW_BN) &&
+            make_g_map(&tg, gbase, N, M, batch, epi.ldrow, epi.ldG)) {
+            e = bk == 64 ? launch_dw<64, 3>(ta, tb, tg, M, N, K, batch, status, st)
+                         : launch_dw<32, 4>(ta, tb, tg, M, N, K, batch, status, st);
+            if (e != cudaSuccess) return fail(DBW_ECUDA, "tc_gemm launch: %s", cudaGetErrorString(e));
+            return DBW_OK;
+        }
         if (!make_map(&ta, A, rowsA, colsA, lda, bk, BM) || !make_map(&tb, B, rowsB, colsB, ldb, bk, 128))
             return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
         // 4 CTAs per SM (48 KB of shared memory each) share the 512 TMEM columns, 128 each
