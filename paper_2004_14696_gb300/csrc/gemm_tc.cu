@@ -134,23 +134,11 @@ __host__ __device__ constexpr uint32_t instr_desc_bf16(int m, int n) {
 
 __device__ __forceinline__ float u2f(uint32_t u) { return __uint_as_float(u); }
 
-// TMA bulk tensor store (shared -> global) of a 3-D box, and its bulk-group bookkeeping.
-__device__ __forceinline__ void tma_store_3d(const CUtensorMap* tm, uint32_t src, int x, int y, int z) {
-    asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
-                     reinterpret_cast<uint64_t>(tm)),
-                 "r"(src), "r"(x), "r"(y), "r"(z)
+// 32-byte streaming store of eight fp32 values (a whole L2 sector); p 32-byte aligned.
+__device__ __forceinline__ void st_v8_stream(float* p, const uint32_t* v) {
+    asm volatile("st.global.cs.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(v[0]), "r"(v[1]), "r"(v[2]),
+                 "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
                  : "memory");
-}
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-// wait until at most N committed bulk groups of this thread still read shared memory
-template <int N>
-__device__ __forceinline__ void bulk_wait_read() {
-    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
-}
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-// make this thread's generic-proxy shared-memory writes visible to the async proxy (TMA)
-__device__ __forceinline__ void fence_proxy_async_smem() {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
@@ -233,19 +221,11 @@ __device__ __forceinline__ void epilogue_chunk(const TcEpi& e, int z, int row, i
             for (int j = 0; j < 32; ++j)
                 if (nb + j < N) op[j] = u2f(r[j]) + __ldg(e.bias + nb + j);
         }
-    } else {   // TC_DW
+    } else {   // TC_DW: element (m, n) -> G[z*ldG + off + m*ldrow + n]
         float* op = e.G + static_cast<int64_t>(z) * e.ldG + e.off + static_cast<int64_t>(row) * e.ldrow + nb;
-        if (full && ((reinterpret_cast<uintptr_t>(op) & 15u) == 0)) {
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                float4 v = make_float4(u2f(r[4 * q]), u2f(r[4 * q + 1]), u2f(r[4 * q + 2]), u2f(r[4 * q + 3]));
-                __stcs(reinterpret_cast<float4*>(op + 4 * q), v);   // streaming: G is read back much later
-            }
-        } else {
-#pragma unroll
-            for (int j = 0; j < 32; ++j)
-                if (nb + j < N) op[j] = u2f(r[j]);
-        }
+        for (int j = 0; j < 32; ++j)
+            if (nb + j < N) __stcs(op + j, u2f(r[j]));
     }
 }
 
@@ -372,16 +352,23 @@ __global__ void __launch_bounds__(kThreads, MINB)
 }
 
 // ------------------------------------------------------------------ persistent dW kernel
-// Per-worker weight gradient G[z, off + m*ldrow + n] = sum_{k < K} A[m, z*K + k] B[n, z*K + k]
-// (A = dZ^T [out, M], B = A_{l-1}^T [in, M], K = B samples), written by TMA bulk
-// stores.  The kernel is bound by writing G (K is small), so it is built around
-// the store: a persistent grid (one CTA per SM) walks the tiles (worker-major),
-// the MMA of tile i+1 runs into the second of two 256-column TMEM accumulators
-// while the epilogue drains tile i, and each epilogue warp moves its 32 x 32 fp32
-// chunks TMEM -> registers -> 128B-swizzled shared memory (conflict-free) -> one
-// TMA store, double-buffered.
+// Per-worker weight gradient G[z*ldG + m*ldrow + n] = sum_{k < K} A[m, z*K + k] B[n, z*K + k]
+// (A = dZ^T [out, M], B = A_{l-1}^T [in, M], K = the worker's B samples).
+//
+// The kernel is bound by writing G (K is small), so it is built around that
+// store.  A persistent grid (one CTA per SM) walks the tiles worker-major with n
+// fastest; the MMA of tile i+1 runs into the second of two 256-column TMEM
+// accumulators while the epilogue drains tile i.  Eight epilogue warps: two per
+// TMEM lane quarter (32 rows of G), each owning 128 of the tile's 256 columns.
+// A warp copies its 32 x 128 fp32 block TMEM -> registers -> shared memory
+// (16-byte pieces XOR-swizzled by row, conflict-free) and then writes it row by
+// row: each store instruction covers 512 contiguous bytes of one G row, the
+// pattern that reaches the highest write bandwidth on this part.
 constexpr int DW_BN = 256;
-constexpr int DW_CHUNK_BYTES = 32 * 32 * 4;   // one warp's 32 rows x 32 fp32 columns
+constexpr int DW_EPI_WARPS = 8;
+constexpr int DW_THREADS = 32 * (2 + DW_EPI_WARPS);
+constexpr int DW_WARP_COLS = 128;                         // columns of the tile per epilogue warp
+constexpr int DW_STAGING_BYTES = 32 * DW_WARP_COLS * 4;   // 32 rows x 512 bytes per warp
 
 template <int BK, int STAGES>
 struct DwCfg {
@@ -389,25 +376,25 @@ struct DwCfg {
     static constexpr int B_BYTES = DW_BN * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr int SW = BK * 2;
-    static constexpr int STAGING = 4 * 2 * DW_CHUNK_BYTES;   // 4 epilogue warps x 2 buffers
+    static constexpr int STAGING = DW_EPI_WARPS * DW_STAGING_BYTES;
     static constexpr int BAR_BYTES = 256;
     static constexpr int SMEM = STAGES * STAGE_BYTES + STAGING + BAR_BYTES + 1024;
 };
 
 template <int BK, int STAGES>
-__global__ void __launch_bounds__(kThreads, 1)
-    tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                 const __grid_constant__ CUtensorMap tmG, int Mr, int Nr, int K, int batch, int* status) {
+__global__ void __launch_bounds__(DW_THREADS, 1)
+    tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int Mr, int Nr,
+                 int K, int batch, int* status, float* __restrict__ Gbase, int64_t ldrow, int64_t ldG) {
     using Cfg = DwCfg<BK, STAGES>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sA = smem;
     uint8_t* sB = smem + STAGES * Cfg::A_BYTES;
-    uint8_t* stage_out = smem + STAGES * Cfg::STAGE_BYTES;   // 1024-aligned (stage sizes are)
-    uint64_t* full_bar = reinterpret_cast<uint64_t*>(stage_out + Cfg::STAGING);
+    uint8_t* staging = smem + STAGES * Cfg::STAGE_BYTES;
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(staging + Cfg::STAGING);
     uint64_t* empty_bar = full_bar + STAGES;
     uint64_t* tfull_bar = empty_bar + STAGES;    // [2] accumulator ready
-    uint64_t* tempty_bar = tfull_bar + 2;        // [2] accumulator drained (4 epilogue warps)
+    uint64_t* tempty_bar = tfull_bar + 2;        // [2] accumulator drained (all epilogue warps)
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty_bar + 2);
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
@@ -424,7 +411,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(smem_u32(tfull_bar + a), 1);
-            mbar_init(smem_u32(tempty_bar + a), 4);
+            mbar_init(smem_u32(tempty_bar + a), DW_EPI_WARPS);
         }
         *abort_flag = 0;
         fence_mbar_init();
@@ -446,6 +433,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (long long t = blockIdx.x; t < total && !*vabort; t += gridDim.x) {
             const int z = static_cast<int>(t / tiles_per_z);
             const int rem = static_cast<int>(t % tiles_per_z);
+            // n (out) fastest: consecutive tiles, run by neighbouring SMs at the same
+            // time, fill the same G rows' line ranges together
             const int m0 = (rem / nt_n) * BM, n0 = (rem % nt_n) * DW_BN;
             for (int kb = 0; kb < nk; ++kb, ++g) {
                 const int s = static_cast<int>(g % STAGES);
@@ -504,10 +493,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) break;
         }
     } else if (warp >= 2) {
-        // ---------------- epilogue: TMEM -> registers -> swizzled smem -> TMA store
-        const int q = warp & 3;
-        uint8_t* mybuf = stage_out + q * 2 * DW_CHUNK_BYTES;
-        int nbuf = 0;
+        // ---------------- epilogue: TMEM -> registers -> swizzled smem -> 512-byte row stores
+        const int q = warp & 3;                 // TMEM lanes 32q .. 32q+31 = G rows m0 + 32q ..
+        const int half = (warp - 2) >> 2;       // columns [128 half, 128 half + 128) of the tile
+        uint8_t* buf = staging + (warp - 2) * DW_STAGING_BYTES;
         int i = 0;
         for (long long t = blockIdx.x; t < total; t += gridDim.x, ++i) {
             const int acc = i & 1;
@@ -524,37 +513,41 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int m0 = (rem / nt_n) * BM, n0 = (rem % nt_n) * DW_BN;
             const uint32_t tbase = tmem + static_cast<uint32_t>(acc * DW_BN) + (static_cast<uint32_t>(q * 32) << 16);
             const int row0 = m0 + q * 32;
+            const int colw = n0 + half * DW_WARP_COLS;      // first column of this warp's block
+            if (row0 < Mr && colw < Nr) {
+                // 1) TMEM -> smem: lane = row; 16-byte piece p of 128-byte segment sgm of row r
+                //    lives at r*512 + sgm*128 + ((p ^ (r & 7)) * 16)
 #pragma unroll 1
-            for (int c = 0; c < DW_BN / 32; ++c) {
-                const int col0 = n0 + c * 32;
-                if (col0 >= Nr || row0 >= Mr) break;   // whole chunk outside the tensor (warp-uniform)
-                uint32_t r[32];
-                tc_ld_32cols(tbase + c * 32, r);
-                tc_wait_ld();
-                // this buffer was last handed to a TMA store two chunks ago: wait until read
-                if (lane == 0) bulk_wait_read<1>();
-                __syncwarp();
-                uint8_t* buf = mybuf + nbuf * DW_CHUNK_BYTES;
-                // row ``lane``: 8 chunks of 16 bytes, chunk j at (j ^ (lane & 7)) * 16 (128B swizzle)
+                for (int sgm = 0; sgm < DW_WARP_COLS / 32; ++sgm) {
+                    uint32_t r[32];
+                    tc_ld_32cols(tbase + half * DW_WARP_COLS + sgm * 32, r);
+                    tc_wait_ld();
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    uint4 v = make_uint4(r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
-                    *reinterpret_cast<uint4*>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) = v;
+                    for (int pc = 0; pc < 8; ++pc)
+                        *reinterpret_cast<uint4*>(buf + lane * 512 + sgm * 128 + ((pc ^ (lane & 7)) << 4)) =
+                            make_uint4(r[4 * pc], r[4 * pc + 1], r[4 * pc + 2], r[4 * pc + 3]);
                 }
-                fence_proxy_async_smem();
                 __syncwarp();
-                if (lane == 0) {
-                    tma_store_3d(&tmG, smem_u32(buf), col0, row0, z);
-                    bulk_commit();
+                // 2) smem -> G, one row per instruction: lane L writes columns colw + 4L .. +3
+                const int sgm = lane >> 3, pc = lane & 7;
+                const int col = colw + 4 * lane;
+                const bool col_ok = col + 3 < Nr;   // Nr % 4 == 0 on this path: whole pieces in or out
+                float* gcol = Gbase + static_cast<int64_t>(z) * ldG + col;
+#pragma unroll 4
+                for (int rr = 0; rr < 32; ++rr) {
+                    const uint4 v = *reinterpret_cast<const uint4*>(buf + rr * 512 + sgm * 128 + ((pc ^ (rr & 7)) << 4));
+                    if (col_ok && row0 + rr < Mr)
+                        __stcs(reinterpret_cast<float4*>(gcol + static_cast<int64_t>(row0 + rr) * ldrow),
+                               make_float4(__uint_as_float(v.x), __uint_as_float(v.y), __uint_as_float(v.z),
+                                           __uint_as_float(v.w)));
                 }
-                nbuf ^= 1;
+                __syncwarp();
             }
             // every tcgen05.ld of this accumulator has completed (wait::ld above)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(tempty_bar + acc));
         }
-        if (lane == 0) bulk_wait_all();
     }
     tc_fence_before();
     __syncthreads();
@@ -597,31 +590,19 @@ bool make_map(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// 3-D tensor map over the fp32 weight-gradient block of every worker:
-// element (n, m, z) at base + z*ldG + m*ldrow + n, box 32 x 32 x 1, 128B swizzle.
-bool make_g_map(CUtensorMap* tm, const float* base, int64_t Nr, int64_t Mr, int64_t batch, int64_t ldrow,
-                int64_t ldG) {
-    EncodeTiledFn fn = encode_fn();
-    if (!fn) return false;
-    cuuint64_t dims[3] = {static_cast<cuuint64_t>(Nr), static_cast<cuuint64_t>(Mr), static_cast<cuuint64_t>(batch)};
-    cuuint64_t strides[2] = {static_cast<cuuint64_t>(ldrow * 4), static_cast<cuuint64_t>(ldG * 4)};
-    cuuint32_t box[3] = {32, 32, 1};
-    cuuint32_t estr[3] = {1, 1, 1};
-    return fn(tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(base), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 template <int BK, int STAGES>
-cudaError_t launch_dw(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& g, int Mr, int Nr, int K,
-                      int batch, int* status, cudaStream_t st) {
+cudaError_t launch_dw(const CUtensorMap& a, const CUtensorMap& b, int Mr, int Nr, int K, int batch, int* status,
+                      float* gbase, int64_t ldrow, int64_t ldG, cudaStream_t st) {
     using Cfg = DwCfg<BK, STAGES>;
     auto kern = tc_dw_kernel<BK, STAGES>;
-    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    // each CTA holds all 512 TMEM columns: ask for enough shared memory that a
+    // second CTA can never be resident on the same SM (it would wait in tcgen05.alloc)
+    const int smem = Cfg::SMEM > 120 * 1024 ? Cfg::SMEM : 120 * 1024;
+    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (err != cudaSuccess) return err;
     const long long tiles = static_cast<long long>((Mr + BM - 1) / BM) * ((Nr + DW_BN - 1) / DW_BN) * batch;
     const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
-    kern<<<grid, kThreads, Cfg::SMEM, st>>>(a, b, g, Mr, Nr, K, batch, status);
+    kern<<<grid, DW_THREADS, smem, st>>>(a, b, Mr, Nr, K, batch, status, gbase, ldrow, ldG);
     return cudaGetLastError();
 }
 
@@ -657,25 +638,20 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
     if (kind == TC_DW) {
         // K = the per-worker sample count: 64-deep blocks when it allows, else 32
         const int bk = (K % 64 == 0) ? 64 : 32;
-        const float* gbase = epi.G + epi.off;
-        const bool store_ok = ((reinterpret_cast<uintptr_t>(gbase) & 15u) == 0) && (epi.ldrow % 4 == 0) &&
-                              (epi.ldG % 4 == 0) && M >= 1 && N >= 1;
-        CUtensorMap tg;
-        if (store_ok && make_map(&ta, A, rowsA, colsA, lda, bk, BM) &&
-            make_map(&tb, B, rowsB, colsB, ldb, bk, DW_BN) &&
-            make_g_map(&tg, gbase, N, M, batch, epi.ldrow, epi.ldG)) {
-            e = bk == 64 ? launch_dw<64, 3>(ta, tb, tg, M, N, K, batch, status, st)
-                         : launch_dw<32, 4>(ta, tb, tg, M, N, K, batch, status, st);
-            if (e != cudaSuccess) return fail(DBW_ECUDA, "tc_gemm launch: %s", cudaGetErrorString(e));
-            return DBW_OK;
-        }
-        if (!make_map(&ta, A, rowsA, colsA, lda, bk, BM) || !make_map(&tb, B, rowsB, colsB, ldb, bk, 128))
+        if (!make_map(&ta, A, rowsA, colsA, lda, bk, BM) || !make_map(&tb, B, rowsB, colsB, ldb, bk, DW_BN))
             return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
-        // 4 CTAs per SM (48 KB of shared memory each) share the 512 TMEM columns, 128 each
-        if (bk == 64)
-            e = launch_cfg<128, 64, 2, TC_DW, 4>(ta, tb, M, N, K, batch, kz, epi, status, st, 48 * 1024);
-        else
-            e = launch_cfg<128, 32, 2, TC_DW, 4>(ta, tb, M, N, K, batch, kz, epi, status, st, 48 * 1024);
+        float* gb = epi.G + epi.off;
+        const bool vec_ok = ((reinterpret_cast<uintptr_t>(gb) & 15u) == 0) && epi.ldrow % 4 == 0 && epi.ldG % 4 == 0;
+        if (!vec_ok) {
+            // unaligned rows: the one-CTA-per-tile kernel (128-column tiles) with scalar stores
+            if (!make_map(&tb, B, rowsB, colsB, ldb, bk, 128))
+                return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
+            e = bk == 64 ? launch_cfg<128, 64, 2, TC_DW, 4>(ta, tb, M, N, K, batch, kz, epi, status, st, 48 * 1024)
+                         : launch_cfg<128, 32, 2, TC_DW, 4>(ta, tb, M, N, K, batch, kz, epi, status, st, 48 * 1024);
+        } else {
+            e = bk == 64 ? launch_dw<64, 2>(ta, tb, M, N, K, batch, status, gb, epi.ldrow, epi.ldG, st)
+                         : launch_dw<32, 4>(ta, tb, M, N, K, batch, status, gb, epi.ldrow, epi.ldG, st);
+        }
     } else {
         if (!make_map(&ta, A, rowsA, colsA, lda, 64, BM) || !make_map(&tb, B, rowsB, colsB, ldb, 64, 256))
             return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");

@@ -44,7 +44,9 @@ class Workload:
 
     @property
     def ld(self) -> int:
-        return inputs.round_up(self.d, 4)
+        # rows of G start on 128-byte boundaries (the weight-gradient kernel writes
+        # whole 32-byte sectors with 256-bit stores when rows are 32-byte aligned)
+        return inputs.round_up(self.d, 32)
 
     @property
     def classes(self) -> int:
