@@ -47,6 +47,11 @@ UNIT = "iter/s"
 # aggregate.cu differs from the source the counters were taken on.
 AGG_TRAFFIC = {"ratio_to_algorithmic": 793.76e6 / 800.0e6, "source_sha256": "4152d07608f8bd5706924d7da1ef028ddd4243bc397b0c495b09a2b85dba387c",
                "case": "n=64 d=4e6 k=48"}
+# dram bytes (read + write) of the per-worker weight-gradient launches of one
+# full-size step (ncu on mlp4096x3-1000_n256_B32, profiles/tc_dw_kernel_mlp4096_ncu.md):
+# 3 x 17.2562 GB + 4.2130 GB against 3 x 17.3141 GB + 4.2778 GB algorithmic.
+DW_TRAFFIC = {"ratio_to_algorithmic": (3 * 17.2562 + 4.2130) / (3 * 17.3141 + 4.2778),
+              "source_sha256": "92a1a3b4ed63fb66d8df729e0a997fe728dabb3035ebb91bff5addc78a912a76", "case": "mlp4096x3-1000_n256_B32, one step"}
 
 
 def parse():
@@ -83,7 +88,7 @@ class ClockSampler:
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
@@ -197,12 +202,15 @@ def run_dbw(args, rank, world, local_rank):
     torch.cuda.synchronize(dev)
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
+    dbw.dbw_profile_dw(True)
     with ClockSampler(local_rank) as clk:
         t_start.record(stream)
         for t in range(W, total):
             one(t, True)
         t_end.record(stream)
         torch.cuda.synchronize(dev)
+    dw_ms, dw_launches, dw_bytes = dbw.dbw_profile_dw_read()
+    dbw.dbw_profile_dw(False)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
@@ -261,6 +269,19 @@ def run_dbw(args, rank, world, local_rank):
     src = os.path.join(ROOT, "paper_2004_14696_gb300", "csrc", "aggregate.cu")
     if AGG_TRAFFIC["source_sha256"] == sha256_of(src):
         traffic = AGG_TRAFFIC["ratio_to_algorithmic"] * agg_bytes
+    # the dominant kernel (by share of the step): the per-worker weight gradient writing G
+    dw = None
+    if dw_launches:
+        per_bytes, per_ms = dw_bytes / dw_launches, dw_ms / dw_launches
+        dw_ach = per_bytes / (per_ms * 1e-3) / 1e9
+        dsrc = os.path.join(ROOT, "paper_2004_14696_gb300", "csrc", "gemm_tc.cu")
+        dw_traffic = (DW_TRAFFIC["ratio_to_algorithmic"] * per_bytes
+                      if DW_TRAFFIC["source_sha256"] == sha256_of(dsrc) else None)
+        dw = {"kernel": "tc_dw_kernel (per-worker dW GEMM writing G, in dbw_worker_grads)", "bound": "hbm",
+              "achieved": dw_ach, "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": dw_ach / pk["hbm_gbs"],
+              "traffic": dw_traffic, "algorithmic_bytes_per_launch": per_bytes, "ms_per_launch": per_ms,
+              "launches_timed": dw_launches, "share_of_step": dw_ms / K / (elapsed_ms / K),
+              "peak_source": pk["source"]}
     ms_step = elapsed_ms / K
     value = world * K / (elapsed_ms * 1e-3)
     gemm_flop = 0
@@ -278,10 +299,11 @@ def run_dbw(args, rank, world, local_rank):
                    "d": d, "G_bytes": n * it.ld * 4, "time_model": wl.time_model, "policy": "dbw",
                    "mean_k": float(kvals.mean()), "l2": "working set > L2 (G is %.1f GB), no flush"
                    % (n * it.ld * 4 / 1e9), "parallelism": "replicas" if world > 1 else "single"},
-        "roofline": {"kernel": "aggregate_kernel (dbw_aggregate_update)", "bound": "hbm",
-                     "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": achieved / pk["hbm_gbs"],
-                     "traffic": traffic, "algorithmic_bytes_per_launch": agg_bytes,
-                     "peak_source": pk["source"]},
+        "roofline": dw,
+        "roofline_aggregate": {"kernel": "aggregate_kernel (dbw_aggregate_update)", "bound": "hbm",
+                               "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                               "frac": achieved / pk["hbm_gbs"], "traffic": traffic,
+                               "algorithmic_bytes_per_launch": agg_bytes, "peak_source": pk["source"]},
         "phases_ms": phase_ms,
         "gemm": {"flop_per_step": gemm_flop, "worker_grads_tflops": gemm_flop / (phase_ms["worker_grads"] * 1e-3) / 1e12},
         "gpu_launches": None,

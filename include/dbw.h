@@ -168,6 +168,19 @@ int dbw_worker_grads_activations(int num_layers, const int32_t* widths, int n, i
                                  size_t* offset, int64_t* ld, int* elem_bytes);
 
 /*
+ * Opt-in timing of the per-worker weight-gradient launches (the GEMM epilogue
+ * that writes G, the largest HBM stream of an iteration).  While enabled, every
+ * such launch inside dbw_worker_grads is bracketed by CUDA events recorded on
+ * the call's stream.  dbw_profile_dw(enable) turns it on or off and forgets
+ * earlier records; dbw_profile_dw_read waits for the recorded events and returns
+ * the summed launch durations (ms), the number of launches and their summed
+ * algorithmic bytes (G written once in fp32 plus both bf16 operands read once),
+ * then forgets them.  Host only; not for use during stream capture.
+ */
+int dbw_profile_dw(int enable);
+int dbw_profile_dw_read(double* total_ms, int64_t* launches, double* total_bytes);
+
+/*
  * Eq. (4): the PS waits for the first k = n - b gradients.
  * Arrival order is (times[i], i) ascending (ties go to the lower worker index).
  *

@@ -21,6 +21,7 @@
 #include <mutex>
 
 #include "gemm_tc.cuh"
+#include "profile.cuh"
 
 namespace dbw {
 
@@ -638,6 +639,9 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
     if (kind == TC_DW) {
         // K = the per-worker sample count: 64-deep blocks when it allows, else 32
         const int bk = (K % 64 == 0) ? 64 : 32;
+        // algorithmic bytes: G written once (fp32), both bf16 operands read once
+        const double dw_bytes = 4.0 * batch * double(M) * N + 2.0 * batch * double(K) * (double(M) + N);
+        void* prof = dw_profile_begin(st, dw_bytes);
         if (!make_map(&ta, A, rowsA, colsA, lda, bk, BM) || !make_map(&tb, B, rowsB, colsB, ldb, bk, DW_BN))
             return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
         float* gb = epi.G + epi.off;
@@ -652,6 +656,7 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
             e = bk == 64 ? launch_dw<64, 2>(ta, tb, M, N, K, batch, status, gb, epi.ldrow, epi.ldG, st)
                          : launch_dw<32, 4>(ta, tb, M, N, K, batch, status, gb, epi.ldrow, epi.ldG, st);
         }
+        dw_profile_end(prof, st);
     } else {
         if (!make_map(&ta, A, rowsA, colsA, lda, 64, BM) || !make_map(&tb, B, rowsB, colsB, ldb, 64, 256))
             return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");

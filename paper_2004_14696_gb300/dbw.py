@@ -66,6 +66,8 @@ _SIGS = {
     "dbw_state_init": (_i32, [_vp, _i32, _i32, _vp]),
     "dbw_grad_stats": (_i32, [_vp, _i32, _vp, _vp, _vp, _f64, _vp, _vp, _vp, _vp]),
     "dbw_choose_b": (_i32, [_vp, _f64, _f64, _i32, _vp, _vp, _vp]),
+    "dbw_profile_dw": (_i32, [_i32]),
+    "dbw_profile_dw_read": (_i32, [_vp, _vp, _vp]),
 }
 
 
@@ -206,6 +208,17 @@ def dbw_choose_b(state, lr, beta, b_out, ratio_out=None, flags=0, stream=None):
         _ptr(state, torch.uint8, "state"), float(lr), float(beta), int(flags), _ptr(b_out, torch.int32, "b_out"),
         _ptr(ratio_out, torch.float64, "ratio_out", nullable=True), _stream(stream))
     _check("dbw_choose_b", rc)
+
+
+def dbw_profile_dw(enable):
+    _check("dbw_profile_dw", lib().dbw_profile_dw(1 if enable else 0))
+
+
+def dbw_profile_dw_read():
+    """(summed ms, launches, summed algorithmic bytes) of the timed weight-gradient launches."""
+    ms, n, b = C.c_double(), C.c_int64(), C.c_double()
+    _check("dbw_profile_dw_read", lib().dbw_profile_dw_read(C.byref(ms), C.byref(n), C.byref(b)))
+    return ms.value, n.value, b.value
 
 
 # ----------------------------------------------------------------- helpers
