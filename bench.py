@@ -128,6 +128,21 @@ class ClockSampler:
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def combine_over_ranks(values, world, device):
+    """Max over ranks of each per-rank timing: the slowest rank sets the job's time."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def job_value(world, steps, max_elapsed_ms):
+    """Whole-job throughput: every rank ran ``steps`` independent iterations."""
+    return world * steps / (max_elapsed_ms * 1e-3)
+
+
 def sha256_of(path):
     with open(path, "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()
@@ -254,10 +269,7 @@ def run_dbw(args, rank, world, local_rank):
     d2h = stats_pin.numel() * 8
 
     # ---------------------------------------------------------------- gather over ranks
-    mine = torch.tensor([elapsed_ms, e2e_s], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(mine, op=dist.ReduceOp.MAX)
-    elapsed_ms, e2e_s = mine.tolist()
+    elapsed_ms, e2e_s = combine_over_ranks([elapsed_ms, e2e_s], world, dev)
     if rank != 0:
         return None
     pk = peaks()
@@ -283,7 +295,7 @@ def run_dbw(args, rank, world, local_rank):
               "launches_timed": dw_launches, "share_of_step": dw_ms / K / (elapsed_ms / K),
               "peak_source": pk["source"]}
     ms_step = elapsed_ms / K
-    value = world * K / (elapsed_ms * 1e-3)
+    value = job_value(world, K, elapsed_ms)
     gemm_flop = 0
     wd = wl.widths
     M = n * B
@@ -307,7 +319,7 @@ def run_dbw(args, rank, world, local_rank):
         "phases_ms": phase_ms,
         "gemm": {"flop_per_step": gemm_flop, "worker_grads_tflops": gemm_flop / (phase_ms["worker_grads"] * 1e-3) / 1e12},
         "gpu_launches": None,
-        "e2e": {"value": world * K / e2e_s, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+        "e2e": {"value": job_value(world, K, e2e_s * 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h)},
         "clocks": clk.summary(),
     }

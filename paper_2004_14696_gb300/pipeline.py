@@ -86,6 +86,37 @@ class Iteration:
         dbw.dbw_grad_stats(self.partials, wl.n, self.mask, self.loss, self.tsorted, wl.lr, self.state, self.stats,
                            self.row_sqnorm, stream)
 
+    # ------------------------------------------------------------ checkpoint
+    def checkpoint(self):
+        """Host copy of everything an iteration carries over: w and the estimator state.
+
+        The gradient matrix, workspace and partials are scratch that each
+        iteration rewrites, so (w, state) restores the run exactly.
+        """
+        torch.cuda.synchronize(self.device)
+        return {"w": self.w.detach().cpu().clone(), "state": self.state.detach().cpu().clone(),
+                "b": self.b.detach().cpu().clone(), "key": self.wl.key}
+
+    def restore(self, ckpt):
+        if ckpt["key"] != self.wl.key:
+            raise ValueError("checkpoint of another workload")
+        self.w.copy_(ckpt["w"])
+        self.state.copy_(ckpt["state"])
+        self.b.copy_(ckpt["b"])
+
+    def record(self, t, wall_ms=None):
+        """One iteration's log record (reads the statistics back: synchronises)."""
+        s = self.stats.cpu().numpy()
+        st = dbw.read_state(self.state)
+        k = int(s[dbw.STAT_K])
+        rec = {"t": t, "b": self.n - k, "k": k, "T_k": float(self.tsorted[k - 1].item()),
+               "vclock": float(s[dbw.STAT_VCLOCK]), "F": float(s[dbw.STAT_F]),
+               "gbar_sq": float(s[dbw.STAT_GBAR_SQ]), "V": float(s[dbw.STAT_V]), "N": float(s[dbw.STAT_N]),
+               "L": float(s[dbw.STAT_L]), "flags": int(s[dbw.STAT_FLAGS]), "k_next_state": int(st.k_next)}
+        if wall_ms is not None:
+            rec["wall_ms"] = wall_ms
+        return rec
+
     def launches_per_step(self):
         """Kernels libdbw launches per step (for the bench's launch count)."""
         L = len(self.wl.widths) - 1
@@ -107,3 +138,49 @@ def agg_case(n, d, seed, b, device="cuda", mean=0.0, std=1.0):
     w = inputs.rng(seed, inputs.STREAM_INIT).standard_normal(d, dtype=np.float32)
     times = inputs.completion_times(seed, 0, n, "shifted_exp", shift=0.0, rate=1.0)
     return G, w, times
+
+
+def run(wl: Workload, iters, log=None, static_b=None, blind=False, device="cuda", start=0, it=None):
+    """Run ``iters`` iterations of a workload; returns (and optionally writes as JSON
+    lines to the file object ``log``) one record per iteration: b_t, k_t, the k_t-th
+    arrival time T_(k_t) (the iteration's virtual duration), the virtual clock, F^_t,
+    ||g_t||^2, V^+, ||grad F||^2^+, L^+ and the flags raised."""
+    import json
+    import time
+    if it is None:
+        it = Iteration(wl, device=device, static_b=static_b, blind=blind)
+    out = []
+    for t in range(start, start + iters):
+        it.load_inputs(t)
+        t0 = time.perf_counter()
+        it.step()
+        torch.cuda.synchronize(it.device)
+        rec = it.record(t, (time.perf_counter() - t0) * 1e3)
+        out.append(rec)
+        if log is not None:
+            log.write(json.dumps(rec) + "\n")
+    return out, it
+
+
+def _main(argv=None):
+    import argparse
+    import sys
+    from . import workloads
+    p = argparse.ArgumentParser(description="Run a DBW workload and log one JSON line per iteration.")
+    p.add_argument("--workload", default=workloads.MLP784.key, choices=list(workloads.ALL))
+    p.add_argument("--iters", type=int, default=None)
+    p.add_argument("--static-b", type=int, default=None)
+    p.add_argument("--blind", action="store_true", help="B-DBW: the gain of k is k itself")
+    p.add_argument("--log", default="-")
+    a = p.parse_args(argv)
+    wl = workloads.ALL[a.workload]
+    f = sys.stdout if a.log == "-" else open(a.log, "w")
+    try:
+        run(wl, a.iters or wl.iters, f, a.static_b, a.blind)
+    finally:
+        if f is not sys.stdout:
+            f.close()
+
+
+if __name__ == "__main__":
+    _main()
