@@ -352,6 +352,155 @@ __global__ void __launch_bounds__(kThreads, MINB)
     }
 }
 
+// ------------------------------------------------------------------ persistent GEMM kernel
+// The forward and input-gradient GEMMs (K = a layer width: long mainloops) as a
+// persistent kernel: one CTA per SM walks the 128 x 256 output tiles (n
+// fastest, so concurrently running CTAs share the A row block in L2), the TMA
+// ring of STAGES stages runs across tile boundaries, and two 256-column TMEM
+// accumulators let the fused epilogue of tile i (four warps, one per TMEM lane
+// quarter) overlap the mainloop of tile i+1.
+template <int KIND, int STAGES>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_gemm_persistent_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                              int M, int N, int K, TcEpi epi, int* status) {
+    using Cfg = TcCfg<256, 64, STAGES>;
+    constexpr int BN = 256, BK = 64;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sA = smem;
+    uint8_t* sB = smem + STAGES * Cfg::A_BYTES;
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
+    uint64_t* empty_bar = full_bar + STAGES;
+    uint64_t* tfull_bar = empty_bar + STAGES;    // [2]
+    uint64_t* tempty_bar = tfull_bar + 2;        // [2], 4 epilogue warps
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty_bar + 2);
+    int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int mt_n = (M + BM - 1) / BM, nt_n = (N + BN - 1) / BN;
+    const long long total = static_cast<long long>(mt_n) * nt_n;
+    const int nk = (K + BK - 1) / BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(smem_u32(full_bar + s), 1);
+            mbar_init(smem_u32(empty_bar + s), 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(smem_u32(tfull_bar + a), 1);
+            mbar_init(smem_u32(tempty_bar + a), 4);
+        }
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tc_alloc(smem_u32(tmem_slot), 2 * BN);
+        tc_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    volatile int* vabort = abort_flag;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer
+        long long g = 0, issued = 0;
+        for (long long t = blockIdx.x; t < total && !*vabort; t += gridDim.x) {
+            const int m0 = static_cast<int>(t / nt_n) * BM, n0 = static_cast<int>(t % nt_n) * BN;
+            for (int kb = 0; kb < nk; ++kb, ++g) {
+                const int s = static_cast<int>(g % STAGES);
+                const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
+                if (!mbar_wait(smem_u32(empty_bar + s), ph ^ 1)) {
+                    atomicOr(status, 1);
+                    *vabort = 1;
+                    break;
+                }
+                mbar_expect_tx(smem_u32(full_bar + s), Cfg::STAGE_BYTES);
+                tma_load_2d(smem_u32(sA + s * Cfg::A_BYTES), &tmA, kb * BK, m0, smem_u32(full_bar + s));
+                tma_load_2d(smem_u32(sB + s * Cfg::B_BYTES), &tmB, kb * BK, n0, smem_u32(full_bar + s));
+                issued = g + 1;
+            }
+        }
+        if (*vabort) {
+            for (long long q = issued - STAGES < 0 ? 0 : issued - STAGES; q < issued; ++q)
+                mbar_wait(smem_u32(full_bar + q % STAGES), static_cast<uint32_t>((q / STAGES) & 1));
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer
+        constexpr uint32_t idesc = instr_desc_bf16(BM, BN);
+        long long g = 0;
+        int i = 0;
+        for (long long t = blockIdx.x; t < total && !*vabort; t += gridDim.x, ++i) {
+            const int acc = i & 1;
+            const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
+            if (!mbar_wait(smem_u32(tempty_bar + acc), aph ^ 1)) {
+                atomicOr(status, 1);
+                *vabort = 1;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t dcol = tmem + static_cast<uint32_t>(acc * BN);
+            bool ok = true;
+            for (int kb = 0; kb < nk; ++kb, ++g) {
+                const int s = static_cast<int>(g % STAGES);
+                const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
+                if (!mbar_wait(smem_u32(full_bar + s), ph)) {
+                    atomicOr(status, 1);
+                    *vabort = 1;
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t a0 = smem_u32(sA + s * Cfg::A_BYTES);
+                const uint32_t b0 = smem_u32(sB + s * Cfg::B_BYTES);
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk)
+                    tc_mma(dcol, smem_desc(a0 + kk * 32, Cfg::SW), smem_desc(b0 + kk * 32, Cfg::SW), idesc,
+                           (kb > 0 || kk > 0) ? 1u : 0u);
+                tc_commit(smem_u32(empty_bar + s));
+            }
+            tc_commit(smem_u32(tfull_bar + acc));
+            if (!ok) break;
+        }
+    } else if (warp >= 2) {
+        // ---------------- epilogue
+        const int q = warp & 3;
+        int i = 0;
+        for (long long t = blockIdx.x; t < total; t += gridDim.x, ++i) {
+            const int acc = i & 1;
+            const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
+            if (!mbar_wait(smem_u32(tfull_bar + acc), aph)) {
+                atomicOr(status, 1);
+                *vabort = 1;
+                break;
+            }
+            if (*vabort) break;
+            tc_fence_after();
+            const int m0 = static_cast<int>(t / nt_n) * BM, n0 = static_cast<int>(t % nt_n) * BN;
+            const int row = m0 + q * 32 + lane;
+            const uint32_t tbase = tmem + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
+#pragma unroll 1
+            for (int c = 0; c < BN / 32; ++c) {
+                if (n0 + c * 32 >= N) break;
+                uint32_t r[32];
+                tc_ld_32cols(tbase + c * 32, r);
+                tc_wait_ld();
+                epilogue_chunk<KIND>(epi, 0, row, n0 + c * 32, M, N, r);
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(tempty_bar + acc));
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tc_dealloc(tmem, 2 * BN);
+    }
+}
+
 // ------------------------------------------------------------------ persistent dW kernel
 // Per-worker weight gradient G[z*ldG + m*ldrow + n] = sum_{k < K} A[m, z*K + k] B[n, z*K + k]
 // (A = dZ^T [out, M], B = A_{l-1}^T [in, M], K = the worker's B samples).
@@ -607,6 +756,20 @@ cudaError_t launch_dw(const CUtensorMap& a, const CUtensorMap& b, int Mr, int Nr
     return cudaGetLastError();
 }
 
+template <int KIND>
+cudaError_t launch_persistent(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, const TcEpi& e,
+                              int* status, cudaStream_t st) {
+    constexpr int STAGES = 4;
+    using Cfg = TcCfg<256, 64, STAGES>;
+    auto kern = tc_gemm_persistent_kernel<KIND, STAGES>;
+    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
+    if (err != cudaSuccess) return err;
+    const long long tiles = static_cast<long long>((M + BM - 1) / BM) * ((N + 255) / 256);
+    const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
+    kern<<<grid, kThreads, Cfg::SMEM, st>>>(a, b, M, N, K, e, status);
+    return cudaGetLastError();
+}
+
 template <int BN, int BK, int STAGES, int KIND, int MINB>
 cudaError_t launch_cfg(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, int batch, int64_t kz,
                        const TcEpi& e, int* status, cudaStream_t st, int min_smem) {
@@ -660,13 +823,13 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
     } else {
         if (!make_map(&ta, A, rowsA, colsA, lda, 64, BM) || !make_map(&tb, B, rowsB, colsB, ldb, 64, 256))
             return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
-        // one CTA per SM (4 stages x 48 KB), 256 TMEM columns
+        // persistent: one CTA per SM (4 stages x 48 KB), 2 x 256 TMEM columns
         if (kind == TC_HIDDEN)
-            e = launch_cfg<256, 64, 4, TC_HIDDEN, 1>(ta, tb, M, N, K, batch, kz, epi, status, st, 0);
+            e = launch_persistent<TC_HIDDEN>(ta, tb, M, N, K, epi, status, st);
         else if (kind == TC_LOGITS)
-            e = launch_cfg<256, 64, 4, TC_LOGITS, 1>(ta, tb, M, N, K, batch, kz, epi, status, st, 0);
+            e = launch_persistent<TC_LOGITS>(ta, tb, M, N, K, epi, status, st);
         else
-            e = launch_cfg<256, 64, 4, TC_DX, 1>(ta, tb, M, N, K, batch, kz, epi, status, st, 0);
+            e = launch_persistent<TC_DX>(ta, tb, M, N, K, epi, status, st);
     }
     if (e != cudaSuccess) return fail(DBW_ECUDA, "tc_gemm launch: %s", cudaGetErrorString(e));
     return DBW_OK;
