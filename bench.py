@@ -76,7 +76,7 @@ def peaks():
 
 class ClockSampler:
     """nvidia-smi clock / throttle samples while the timed region runs."""
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    Q = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -84,6 +84,7 @@ class ClockSampler:
         self.gpu = gpu_index
         self.proc = None
         self.lines = []
+        self.window = None       # (start, end) wall-clock seconds of the timed region
 
     def __enter__(self):
         try:
@@ -98,7 +99,10 @@ class ClockSampler:
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.time(), line.strip()))
+
+    def mark(self, start, end):
+        self.window = (start, end)
 
     def __exit__(self, *a):
         if self.proc is not None:
@@ -109,23 +113,38 @@ class ClockSampler:
                 self.proc.kill()
 
     def summary(self):
-        sm, mx, reasons = [], None, set()
+        """Median SM clock and throttle reasons of the samples taken during the timed
+        window (a sample's arrival time is within 100 ms of the window); if the window
+        is shorter than the sampling period, the samples nearest to it."""
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in self.lines:
+        parsed = []
+        for (arrival, line) in self.lines:
             f = [x.strip() for x in line.split(",")]
-            if len(f) < 9:
+            if len(f) < 10:
                 continue
             try:
-                sm.append(float(f[1]))
-                mx = float(f[2])
+                parsed.append((arrival, float(f[2]), float(f[3]), f[6:10]))
             except ValueError:
                 continue
-            for name, v in zip(names, f[5:9]):
+        if not parsed:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        chosen = parsed
+        where = "whole run"
+        if self.window:
+            a, b = self.window
+            inside = [p for p in parsed if a - 0.1 <= p[0] <= b + 0.1]
+            if inside:
+                chosen, where = inside, "timed region"
+            else:
+                mid = 0.5 * (a + b)
+                chosen, where = sorted(parsed, key=lambda p: abs(p[0] - mid))[:2], "nearest to timed region"
+        reasons = set()
+        for p in chosen:
+            for name, v in zip(names, p[3]):
                 if v.lower().startswith("active"):
                     reasons.add(name)
-        if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+        return {"sm_mhz": statistics.median(p[1] for p in chosen), "sm_max_mhz": chosen[-1][2],
+                "reasons": sorted(reasons), "samples": len(chosen), "window": where}
 
 
 def combine_over_ranks(values, world, device):
@@ -150,6 +169,13 @@ def sha256_of(path):
 
 # ====================================================================== DBW arm
 def run_dbw(args, rank, world, local_rank):
+    # nvidia-smi takes a moment to start: the sampler runs for the whole arm, and only
+    # the samples that arrive during the timed region are used
+    with ClockSampler(local_rank) as clk:
+        return _run_dbw(args, rank, world, local_rank, clk)
+
+
+def _run_dbw(args, rank, world, local_rank, clk):
     import torch
     import torch.distributed as dist
 
@@ -218,12 +244,14 @@ def run_dbw(args, rank, world, local_rank):
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     dbw.dbw_profile_dw(True)
-    with ClockSampler(local_rank) as clk:
-        t_start.record(stream)
-        for t in range(W, total):
-            one(t, True)
-        t_end.record(stream)
-        torch.cuda.synchronize(dev)
+    wall0 = time.time()
+    t_start.record(stream)
+    for t in range(W, total):
+        one(t, True)
+    t_end.record(stream)
+    torch.cuda.synchronize(dev)
+    clk.mark(wall0, time.time())
+    time.sleep(0.15)                # let the sampler deliver the samples of the window
     dw_ms, dw_launches, dw_bytes = dbw.dbw_profile_dw_read()
     dbw.dbw_profile_dw(False)
     if world > 1:
