@@ -66,6 +66,17 @@ def label_pool(seed: int, S: int, classes: int) -> np.ndarray:
     return rng(seed, STREAM_LABELS).integers(0, classes, size=S, dtype=np.int32)
 
 
+def teacher_labels(seed: int, X: np.ndarray, classes: int, chunk_rows: int = 8192) -> np.ndarray:
+    """Learnable labels [S] int32: argmax over classes of X @ T, with T ~ N(0,1) [dim, classes]
+    a fixed seeded "teacher" map (a task a classifier can actually fit, so that
+    training losses fall steadily instead of fluctuating around log(classes))."""
+    T = rng(seed, STREAM_LABELS, 1).standard_normal((X.shape[1], classes)).astype(np.float32)
+    out = np.empty(X.shape[0], dtype=np.int32)
+    for c0 in range(0, X.shape[0], chunk_rows):
+        out[c0:c0 + chunk_rows] = np.argmax(X[c0:c0 + chunk_rows] @ T, axis=1)
+    return out
+
+
 # --------------------------------------------------------------------- model init
 def param_count(widths) -> int:
     """Number of parameters of a fully connected net with these layer widths."""

@@ -79,11 +79,13 @@ class Iteration:
         if self.static_b is None:
             dbw.dbw_choose_b(self.state, wl.lr, wl.beta, self.b, self.ratio,
                              dbw.CHOOSE_BLIND if self.blind else 0, stream)
+        # static b is known on the host: its learning-rate rule applies; DBW uses lr
+        lr = wl.lr if self.static_b is None else wl.lr_for(wl.n - int(self.static_b))
         dbw.dbw_worker_grads(wl.widths, wl.prec, self.w, self.pool, self.labels, idx, wl.n, wl.B, self.G,
                              self.loss, self.ws, stream)
         dbw.dbw_select_fastest(times, self.b, self.order, self.mask, self.tsorted, self.k, stream)
-        dbw.dbw_aggregate_update(self.G, wl.n, self.d, self.mask, wl.lr, self.w, self.partials, self.gbar, stream)
-        dbw.dbw_grad_stats(self.partials, wl.n, self.mask, self.loss, self.tsorted, wl.lr, self.state, self.stats,
+        dbw.dbw_aggregate_update(self.G, wl.n, self.d, self.mask, lr, self.w, self.partials, self.gbar, stream)
+        dbw.dbw_grad_stats(self.partials, wl.n, self.mask, self.loss, self.tsorted, lr, self.state, self.stats,
                            self.row_sqnorm, stream)
 
     # ------------------------------------------------------------ checkpoint

@@ -33,6 +33,15 @@ class Workload:
     beta: float = 1.01
     policy: str = "dbw"      # "dbw" (choose b every iteration) or "static"
     seed_offset: int = 0
+    # learning rate of static-b runs: "fixed" (lr for every k) or "proportional"
+    # (lr * k / n, the rule Sect. 4 uses for static settings); DBW always uses lr
+    lr_rule: str = "fixed"
+
+    def lr_for(self, k: int) -> float:
+        """Learning rate of an iteration that keeps k gradients (static-b runs)."""
+        if self.lr_rule == "proportional":
+            return self.lr * k / self.n
+        return self.lr
 
     @property
     def seed(self) -> int:

@@ -441,3 +441,43 @@ def test_dbw_iterations_independent(wl, iters):
         w_or = w_new
         compared += 1
     assert compared >= 3
+
+
+def test_slowdown_estimator_trajectory_settles_at_half():
+    """Sect. 4.3: all round-trip times equal, then half of the 16 workers 5x slower.
+    Both sides get the same seeded statistics (a loss that falls as Eq. (9) predicts
+    for L = 5, gradient variance small next to the gradient norm) and the slowdown
+    times; b_t is bit-exact on every iteration, k_t = 16 while the times are equal
+    and k_t = n/2 = 8 once the slow half is visible in the time estimates."""
+    n, d, D, lr, beta, t_switch = 16, 4001, 5, 0.05, 1.01, 20
+    rng = np.random.default_rng(7)
+    state = dbw.new_state(n, D)
+    ost = O.State(n=n, D=D)
+    b = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ratio = torch.empty(n, dtype=torch.float64, device="cuda")
+    stats = torch.empty(dbw.STATS_LEN, dtype=torch.float64, device="cuda")
+    ks, F, prev = [], 50.0, None
+    for t in range(60):
+        dbw.dbw_choose_b(state, lr, beta, b, ratio)
+        torch.cuda.synchronize()
+        k, r = O.choose_k(ost, lr, beta)
+        assert n - int(b.item()) == k, t
+        assert same_f64(ratio.cpu().numpy(), r), t
+        ks.append(k)
+        SS = (k - 1) * 0.05 * float(rng.uniform(0.95, 1.05))        # V ~ 0.05 per unit of d
+        g2 = 4.0 + 0.05 / k
+        times = inputs.completion_times(0, t, n, "slowdown", value=1.0, factor=5.0, t_switch=t_switch)
+        if prev is not None:
+            N, V, kk = prev
+            F = F - ((lr - 5 * lr * lr / 2) * N - (5 * lr * lr / 2) * V / kk)
+        loss = np.full(n, F, dtype=np.float32)
+        _, mask, ts = O.select_fastest(times, n - k)
+        SSq, g2q = round(SS * 1024) / 1024.0, round(g2 * 1024) / 1024.0
+        part = seeded_partials(n, 2, SSq, g2q, [1.0 if mask[j] else 0.0 for j in range(n)])
+        dbw.dbw_grad_stats(part, n, dev(mask), dev(loss), dev(ts), lr, state, stats)
+        torch.cuda.synchronize()
+        rec = O.record_iteration(ost, k, SSq, g2q, loss, mask, ts, lr)
+        assert_state_equal(dbw.read_state(state), ost)
+        prev = (rec["N"], rec["V"], k) if k >= 2 else None
+    assert all(k == n for k in ks[2:t_switch]), ks
+    assert all(k == n // 2 for k in ks[t_switch + 2:]), ks

@@ -24,11 +24,13 @@ def built():
     torch.cuda.set_device(0)
 
 
-@pytest.mark.parametrize("b", [0, 5, 15])
-def test_softmax_static_b_trajectory(b):
+@pytest.mark.parametrize("b,rule", [(0, "fixed"), (5, "fixed"), (15, "fixed"), (8, "proportional")])
+def test_softmax_static_b_trajectory(b, rule):
     """Softmax regression (784 -> 10, n = 16, B = 32) with a static number of backup
-    workers: GPU and oracle run 12 iterations each from the same seeds."""
-    wl = workloads.SOFTMAX784
+    workers (and, for one case, the proportional learning-rate rule lr * k / n of
+    Sect. 4): GPU and oracle run 12 iterations each from the same seeds."""
+    from dataclasses import replace
+    wl = replace(workloads.SOFTMAX784, lr_rule=rule)
     it = Iteration(wl, static_b=b, keep_gbar=True)
     pool, labels = it.pool.cpu().numpy(), it.labels.cpu().numpy()
     ost = O.State(n=wl.n, D=wl.D)
@@ -38,7 +40,7 @@ def test_softmax_static_b_trajectory(b):
         it.load_inputs(t)
         it.step()
         torch.cuda.synchronize()
-        ref = O.step(ost, wl.widths, w_or, pool[idx], labels[idx], times, wl.B, wl.lr, wl.beta, b=b)
+        ref = O.step(ost, wl.widths, w_or, pool[idx], labels[idx], times, wl.B, wl.lr_for(wl.n - b), wl.beta, b=b)
         assert np.array_equal(it.mask.cpu().numpy(), ref["mask"])
         assert_worker_grads_match(it.G.cpu().numpy()[:, :wl.d], it.loss.cpu().numpy(), wl.widths, w_or, pool[idx],
                                   labels[idx], wl.B, False, range(wl.n), RTOL_FP32)
