@@ -49,9 +49,10 @@ AGG_TRAFFIC = {"ratio_to_algorithmic": 793.76e6 / 800.0e6, "source_sha256": "415
                "case": "n=64 d=4e6 k=48"}
 # dram bytes (read + write) of the per-worker weight-gradient launches of one
 # full-size step (ncu on mlp4096x3-1000_n256_B32, profiles/tc_dw_kernel_mlp4096_ncu.md):
-# 3 x 17.2562 GB + 4.2130 GB against 3 x 17.3141 GB + 4.2778 GB algorithmic.
-DW_TRAFFIC = {"ratio_to_algorithmic": (3 * 17.2562 + 4.2130) / (3 * 17.3141 + 4.2778),
-              "source_sha256": "92a1a3b4ed63fb66d8df729e0a997fe728dabb3035ebb91bff5addc78a912a76", "case": "mlp4096x3-1000_n256_B32, one step"}
+# 4.2130 + 17.2560 + 17.2543 + 17.2546 GB against 4.2778 + 3 x 17.3141 GB algorithmic;
+# keyed to the dW kernel's own source (dw_source_sha).
+DW_TRAFFIC = {"ratio_to_algorithmic": (4.2130 + 17.2560 + 17.2543 + 17.2546) / (4.2778 + 3 * 17.3141),
+              "source_sha256": "9a7ee52ced946ba0dc44c00873f852f1e90ae35e2f879b1d4e6915a983e936fe", "case": "mlp4096x3-1000_n256_B32, one step"}
 
 
 def parse():
@@ -165,6 +166,25 @@ def job_value(world, steps, max_elapsed_ms):
 def sha256_of(path):
     with open(path, "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()
+
+
+DW_REGION = ("// ------------------------------------------------------------------ persistent dW kernel",
+             "// ------------------------------------------------------------------ host side")
+
+
+def dw_source_sha():
+    """sha256 of the per-worker dW kernel's own source (its region of gemm_tc.cu and the
+    PTX helpers it is built from), so that edits to other kernels of the file keep its
+    traffic record."""
+    csrc = os.path.join(ROOT, "paper_2004_14696_gb300", "csrc")
+    with open(os.path.join(csrc, "gemm_tc.cu")) as f:
+        text = f.read()
+    a, b = text.find(DW_REGION[0]), text.find(DW_REGION[1])
+    if a < 0 or b < a:
+        return None
+    with open(os.path.join(csrc, "tc_ptx.cuh")) as f:
+        helpers = f.read()
+    return hashlib.sha256((text[a:b] + helpers).encode()).hexdigest()
 
 
 # ====================================================================== DBW arm
@@ -296,6 +316,9 @@ def _run_dbw(args, rank, world, local_rank, clk):
     h2d = idx_h[0].nbytes + tim_h[0].nbytes
     d2h = stats_pin.numel() * 8
 
+    # ---------------------------------------------------------------- received form
+    rx = _time_received(wl, dev, idx_d, tim_d, W, K, stream, world)
+
     # ---------------------------------------------------------------- gather over ranks
     elapsed_ms, e2e_s = combine_over_ranks([elapsed_ms, e2e_s], world, dev)
     if rank != 0:
@@ -314,9 +337,8 @@ def _run_dbw(args, rank, world, local_rank, clk):
     if dw_launches:
         per_bytes, per_ms = dw_bytes / dw_launches, dw_ms / dw_launches
         dw_ach = per_bytes / (per_ms * 1e-3) / 1e9
-        dsrc = os.path.join(ROOT, "paper_2004_14696_gb300", "csrc", "gemm_tc.cu")
         dw_traffic = (DW_TRAFFIC["ratio_to_algorithmic"] * per_bytes
-                      if DW_TRAFFIC["source_sha256"] == sha256_of(dsrc) else None)
+                      if DW_TRAFFIC["source_sha256"] == dw_source_sha() else None)
         dw = {"kernel": "tc_dw_kernel (per-worker dW GEMM writing G, in dbw_worker_grads)", "bound": "hbm",
               "achieved": dw_ach, "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": dw_ach / pk["hbm_gbs"],
               "traffic": dw_traffic, "algorithmic_bytes_per_launch": per_bytes, "ms_per_launch": per_ms,
@@ -352,6 +374,80 @@ def _run_dbw(args, rank, world, local_rank, clk):
         "clocks": clk.summary(),
     }
     out["gpu_launches"] = it.launches_per_step() * K
+    if rx is not None:
+        kk = rx.pop("_k")
+        flop = 0
+        for l in range(len(wd) - 1):
+            flop += 2 * kk * B * wd[l] * wd[l + 1] * (3 if l > 0 else 2)   # forward, g_t GEMM, input gradient
+        t_upd = rx["phases_ms"]["received_update"] * 1e-3
+        rx["tensor"] = {"flop_per_step": flop, "tflops": flop / t_upd / 1e12,
+                        "frac_of_sustained": flop / t_upd / 1e12 / pk["bf16_tflops_sustained"]
+                        if pk.get("bf16_tflops_sustained") else None,
+                        "peak_sustained": pk.get("bf16_tflops_sustained"), "peak_source": pk["source"]}
+        out["received_form"] = rx
+    return out
+
+
+def _time_received(wl, dev, idx_d, tim_d, W, K, stream, world):
+    """The same iterations in the received-workers form (dbw_received_grads_update: no
+    [n, d] matrix, gradients of the k received workers only), timed the same way."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2004_14696_gb300 import dbw
+    from paper_2004_14696_gb300.pipeline import Iteration
+
+    if dbw.dbw_received_grads_workspace_bytes(wl.widths, wl.n, wl.B, wl.prec) == 0:
+        return None
+    it = Iteration(wl, device=dev, received=True)
+    n, B = wl.n, wl.B
+    total = W + K
+    names = ["choose_b", "select", "received_update", "grad_stats"]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)] for _ in range(total)]
+    ks = torch.zeros(total, dtype=torch.int32, device=dev)
+
+    def one(t, timed):
+        e = ev[t]
+        if timed:
+            e[0].record(stream)
+        dbw.dbw_choose_b(it.state, wl.lr, wl.beta, it.b, it.ratio, 0, stream)
+        if timed:
+            e[1].record(stream)
+        dbw.dbw_select_fastest(tim_d[t], it.b, it.order, it.mask, it.tsorted, it.k, stream)
+        if timed:
+            e[2].record(stream)
+        dbw.dbw_received_grads_update(wl.widths, wl.prec, it.w, it.pool, it.labels, idx_d[t], n, B, it.mask, wl.lr,
+                                      it.loss, it.partials, it.ws, None, stream)
+        if timed:
+            e[3].record(stream)
+        dbw.dbw_grad_stats(it.partials, n, it.mask, it.loss, it.tsorted, wl.lr, it.state, it.stats, it.row_sqnorm,
+                           stream)
+        if timed:
+            e[4].record(stream)
+        ks[t:t + 1].copy_(it.k)
+
+    for t in range(W):
+        one(t, False)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for t in range(W, total):
+        one(t, True)
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = t0.elapsed_time(t1)
+    (ms,) = combine_over_ranks([ms], world, dev)
+    phase = {nm: sum(ev[t][i].elapsed_time(ev[t][i + 1]) for t in range(W, total)) / K for i, nm in enumerate(names)}
+    kv = ks[W:].cpu().numpy().astype(np.float64)
+    status = int(it.ws[:4].view(torch.int32).item())
+    out = {"call": "dbw_received_grads_update", "value": job_value(world, K, ms), "unit": UNIT,
+           "ms_per_step": ms / K, "phases_ms": phase, "mean_k": float(kv.mean()), "device_status": status,
+           "gpu_launches": it.launches_per_step() * K, "_k": float(kv.mean())}
+    del it
+    torch.cuda.empty_cache()
     return out
 
 

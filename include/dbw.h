@@ -13,6 +13,11 @@
  *   dbw_grad_stats        Eqs. (10)-(12) and Sect. 3.2: finishes the statistics
  *                         and records them (and the order statistics) in the state
  *
+ * A second form of the iteration skips the [n, d] matrix:
+ *   dbw_received_grads_update  Eqs. (2)-(4) and the partial sums of Eqs. (10)-(11)
+ *                         for the received workers only (replaces dbw_worker_grads +
+ *                         dbw_aggregate_update after dbw_select_fastest)
+ *
  * Conventions shared by every call:
  *  - Every pointer argument is a DEVICE pointer owned by the caller unless its
  *    comment says "host".  The library never allocates in these calls; scratch
@@ -266,6 +271,63 @@ int dbw_aggregate_update(const float* G, int64_t ld, int n, int64_t d,
 int dbw_aggregate_update_noalloc(const float* G, int64_t ld, int n, int64_t d, const uint8_t* mask, float lr,
                                  float* w, float* gbar, double* sums_out, void* stream);
 
+/* Workspace bytes dbw_received_grads_update needs for (widths, n, B, prec); 0 if
+ * the shape is invalid or the call does not support it. */
+size_t dbw_received_grads_workspace_bytes(int num_layers, const int32_t* widths, int n, int B, int prec);
+
+/* Bytes of the partials buffer dbw_received_grads_update writes for n workers
+ * (the layout above with blocks = 1). */
+size_t dbw_received_partials_bytes(int n);
+
+/*
+ * One PS iteration for the k received workers without the [n, d] gradient
+ * matrix: the same w_{t+1} and statistics as dbw_worker_grads followed by
+ * dbw_aggregate_update on the rows mask selects, computed as
+ *   Eq. (2) for the received workers only: their minibatches are stacked
+ *     (slot s = the s-th received worker in increasing index order) and the
+ *     forward / backward GEMMs run over those k B rows (under push-and-interrupt,
+ *     Sect. 3, the other workers' gradients are never used);
+ *   Eqs. (3)-(4): g_t(W_l) = (1/k) dZ_l^T A_{l-1} over the k B stacked rows, one
+ *     GEMM with K = k B whose epilogue applies w -= lr g_t; the bias part is the
+ *     mean of the per-worker column sums of dZ_l;
+ *   ||g_j||^2 of every received worker from two B x B Gram matrices per layer,
+ *     ||dZ_j^T A_j||^2 + ||1^T dZ_j||^2 = <dZ_j dZ_j^T, A_j A_j^T + 1 1^T>
+ *     (never forming g_j);
+ *   the deviation sum of Eq. (10) by sum_j ||g_j - g_t||^2 = sum_j ||g_j||^2
+ *     - k ||g_t||^2 in fp64, and ||g_t||^2, into ``partials``, which the next
+ *     dbw_grad_stats reduces exactly as after dbw_aggregate_update.
+ * The tensor cores carry the weight-gradient work (K = k B instead of B), and the
+ * n d fp32 writes and k d reads of G disappear.  Rounding differs from the
+ * two-call form: the mean is an fp32 tensor-core sum over k B rows, the norms come
+ * from fp32 Gram entries, and the deviation sum is a difference, whose relative
+ * error grows as sum_j ||g_j||^2 / SS.
+ *
+ *  num_layers, widths, pool, S, labels, idx, n, B   as for dbw_worker_grads.
+ *  prec    DBW_PREC_BF16 only, with B % 32 == 0 and (128 % B == 0 or B % 128 == 0);
+ *          anything else returns DBW_EUNSUPPORTED.
+ *  w       [d] fp32 parameters, updated in place to w_{t+1} (16-byte aligned).
+ *  mask    [n] uint8 from dbw_select_fastest; k = number of set bytes, counted on
+ *          the device.  With k = 0 nothing is updated and the sums are NaN.
+ *  lr      the step eta of Eq. (4).
+ *  gbar    [d] fp32 out (nullable, 16-byte aligned): g_t.
+ *  loss    [n] fp32 out: minibatch mean loss of each received worker; NaN for
+ *          the workers mask leaves out (their loss is never computed).
+ *  partials  [partials_bytes >= dbw_received_partials_bytes(n)], 256-byte aligned.
+ *  ws      workspace of ws_bytes >= dbw_received_grads_workspace_bytes(...),
+ *          256-byte aligned; its first 4 bytes hold the status word of
+ *          dbw_worker_grads (bit 0: a bounded tensor-core wait timed out; the
+ *          outputs are then undefined).  The activations of layer ``layer`` are
+ *          where dbw_worker_grads_activations(..., DBW_PREC_BF16, ...) says, with
+ *          slot s at rows s B .. s B + B - 1 (rows of slots >= k are scratch).
+ */
+int dbw_received_grads_update(int num_layers, const int32_t* widths, int prec,
+                              float* w, int64_t d,
+                              const float* pool, int64_t S, const int32_t* labels,
+                              const int32_t* idx, int n, int B,
+                              const uint8_t* mask, float lr, float* gbar, float* loss,
+                              double* partials, size_t partials_bytes,
+                              void* ws, size_t ws_bytes, void* stream);
+
 /* Initialise a device dbw_state for n workers and window D (k_0 = n). */
 int dbw_state_init(dbw_state* state, int n, int D, void* stream);
 
@@ -278,7 +340,8 @@ int dbw_state_init(dbw_state* state, int n, int D, void* stream);
  * recorded into the state's rings (k = 1 and invalid Eq. (12) values are not
  * recorded), S[r] += tsorted[r] for all r, c += 1, vclock += tsorted[k-1].
  *
- *  partials    the buffer the preceding dbw_aggregate_update of this iteration wrote.
+ *  partials    the buffer the preceding dbw_aggregate_update (or
+ *              dbw_received_grads_update) of this iteration wrote.
  *  mask, loss  [n] this iteration's selection and per-worker losses.
  *  tsorted     [n] from dbw_select_fastest.
  *  lr          the learning rate eta used by the update.

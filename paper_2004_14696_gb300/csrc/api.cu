@@ -145,6 +145,39 @@ int dbw_aggregate_update(const float* G, int64_t ld, int n, int64_t d, const uin
     return DBW_OK;
 }
 
+size_t dbw_received_grads_workspace_bytes(int num_layers, const int32_t* widths, int n, int B, int prec) {
+    if (!widths) return 0;
+    return received_workspace_bytes(num_layers, widths, n, B, prec);
+}
+
+size_t dbw_received_partials_bytes(int n) {
+    if (n < 1 || n > DBW_NMAX) return 0;
+    return sizeof(double) * (kPartialsHeader + 2 * ((size_t)n + 2));
+}
+
+int dbw_received_grads_update(int num_layers, const int32_t* widths, int prec, float* w, int64_t d, const float* pool,
+                              int64_t S, const int32_t* labels, const int32_t* idx, int n, int B, const uint8_t* mask,
+                              float lr, float* gbar, float* loss, double* partials, size_t partials_bytes, void* ws,
+                              size_t ws_bytes, void* stream) {
+    g_err[0] = 0;
+    if (!widths || !w || !pool || !labels || !idx || !mask || !loss || !partials || !ws)
+        return fail(DBW_EINVAL, "dbw_received_grads_update: NULL pointer argument");
+    if (S < 1) return fail(DBW_EINVAL, "dbw_received_grads_update: S must be >= 1");
+    if (n < 1 || n > DBW_NMAX) return fail(DBW_EINVAL, "dbw_received_grads_update: n must be in [1, %d]", DBW_NMAX);
+    if (partials_bytes < dbw_received_partials_bytes(n))
+        return fail(DBW_EINVAL, "dbw_received_grads_update: partials %zu bytes < %zu needed", partials_bytes,
+                    dbw_received_partials_bytes(n));
+    if (!aligned16(w) || !aligned16(pool) || (gbar && !aligned16(gbar)) || !aligned256(partials) || !aligned256(ws))
+        return fail(DBW_EALIGN,
+                    "dbw_received_grads_update: w, pool, gbar must be 16-byte and partials, ws 256-byte aligned");
+    if (num_layers >= 1 && num_layers <= DBW_LMAX && widths[0] % 4 != 0)
+        return fail(DBW_EALIGN, "dbw_received_grads_update: widths[0] must be a multiple of 4");
+    int rc = check_device();
+    if (rc) return rc;
+    return launch_received_grads(num_layers, widths, prec, w, d, pool, S, labels, idx, n, B, mask, lr, gbar, loss,
+                                 partials, ws, ws_bytes, as_stream(stream));
+}
+
 int dbw_state_init(dbw_state* state, int n, int D, void* stream) {
     g_err[0] = 0;
     if (!state) return fail(DBW_EINVAL, "dbw_state_init: NULL state");

@@ -56,7 +56,13 @@ int launch_worker_grads(int L, const int32_t* widths, int prec, const float* w, 
                         int n, int B, float* G, int64_t ld, float* loss, void* ws, size_t ws_bytes,
                         cudaStream_t st);
 
-// Partials buffer layout shared by aggregate.cu and estimator.cu:
+// Received-workers pass (grads_tc.cu)
+size_t received_workspace_bytes(int L, const int32_t* widths, int n, int B, int prec);
+int launch_received_grads(int L, const int32_t* widths, int prec, float* w, int64_t d, const float* pool, int64_t S,
+                          const int32_t* labels, const int32_t* idx, int n, int B, const uint8_t* mask, float lr,
+                          float* gbar, float* loss, double* partials, void* ws, size_t ws_bytes, cudaStream_t st);
+
+// Partials buffer layout shared by aggregate.cu, grads_tc.cu and estimator.cu:
 //   int64 header[4] = {magic, blocks, n, reserved}
 //   double sums[n + 2]              reduced totals (written by dbw_grad_stats)
 //   double vals[(n + 2) * blocks]   per-block pieces, by quantity: vals[q * blocks + blk]

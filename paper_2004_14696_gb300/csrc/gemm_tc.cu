@@ -22,133 +22,16 @@
 
 #include "gemm_tc.cuh"
 #include "profile.cuh"
+#include "tc_ptx.cuh"
 
 namespace dbw {
 
 namespace {
 
+using namespace tcx;
+
 constexpr int BM = 128;
 constexpr int kThreads = 192;
-constexpr uint64_t kWaitLimitNs = 2000000000ull;
-
-// ------------------------------------------------------------------ PTX wrappers
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-__device__ __forceinline__ uint64_t globaltimer() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-// Bounded wait for the phase of parity ``parity`` to complete.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = globaltimer();
-    while (!mbar_try_wait(bar, parity))
-        if (globaltimer() - t0 > kWaitLimitNs) return false;
-    return true;
-}
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm, int x, int y, uint32_t bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
-            dst),
-        "l"(reinterpret_cast<uint64_t>(tm)), "r"(bar), "r"(x), "r"(y)
-        : "memory");
-}
-__device__ __forceinline__ void tc_alloc(uint32_t slot, uint32_t ncols) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(slot), "r"(ncols) : "memory");
-}
-__device__ __forceinline__ void tc_relinquish() {
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void tc_dealloc(uint32_t taddr, uint32_t ncols) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_mma(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
-        "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-__device__ __forceinline__ void tc_commit(uint32_t bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ void tc_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-// 32 consecutive fp32 columns of this thread's TMEM lane.
-__device__ __forceinline__ void tc_ld_32cols(uint32_t taddr, uint32_t (&r)[32]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr));
-}
-
-// UMMA shared-memory matrix descriptor for a K-major operand staged by TMA with
-// a ``sw``-byte swizzle (rows of sw bytes, 8-row atoms).  Fields: start address
-// >> 4 (bits 0-13), leading-dimension offset (unused for swizzled K-major, 1),
-// stride between 8-row groups >> 4 (bits 32-45), descriptor version 1 (bit 46),
-// base offset 0 (tiles are atom aligned), swizzle mode (bits 61-63:
-// 2 = 128B, 4 = 64B).
-__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, int sw) {
-    uint64_t d = 0;
-    d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
-    d |= static_cast<uint64_t>(1) << 16;
-    d |= static_cast<uint64_t>((8u * sw) >> 4) << 32;
-    d |= static_cast<uint64_t>(1) << 46;
-    d |= static_cast<uint64_t>(sw == 128 ? 2 : 4) << 61;
-    return d;
-}
-
-// Instruction descriptor of kind::f16: D fp32 (bits 4-5 = 1), A and B bf16
-// (bits 7-9 = 1, 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at bit 17,
-// M >> 4 at bit 24.
-__host__ __device__ constexpr uint32_t instr_desc_bf16(int m, int n) {
-    return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(n >> 3) << 17) |
-           (static_cast<uint32_t>(m >> 4) << 24);
-}
-
-__device__ __forceinline__ float u2f(uint32_t u) { return __uint_as_float(u); }
-
-// 32-byte streaming store of eight fp32 values (a whole L2 sector); p 32-byte aligned.
-__device__ __forceinline__ void st_v8_stream(float* p, const uint32_t* v) {
-    asm volatile("st.global.cs.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(v[0]), "r"(v[1]), "r"(v[2]),
-                 "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
-                 : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
-    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);   // .x = a (low half), .y = b
-    return *reinterpret_cast<const uint32_t*>(&h);
-}
 
 // ------------------------------------------------------------------ epilogues
 // One thread: row ``row`` of the tile, 32 columns starting at ``nb``.
@@ -228,6 +111,46 @@ __device__ __forceinline__ void epilogue_chunk(const TcEpi& e, int z, int row, i
         for (int j = 0; j < 32; ++j)
             if (nb + j < N) __stcs(op + j, u2f(r[j]));
     }
+}
+
+// GBAR: one thread, row ``row`` (an output unit), 32 columns from ``nb``: the
+// mean over the k received workers, the SGD step and the chunk's sum of squares.
+__device__ __forceinline__ float gbar_chunk(const TcEpi& e, int row, int nb, int M, int N, float inv_k,
+                                            const uint32_t (&r)[32]) {
+    if (row >= M) return 0.f;
+    const int64_t at = e.off + static_cast<int64_t>(row) * e.ldrow + nb;
+    float* wp = e.W + at;
+    float* gp = e.gbar ? e.gbar + at : nullptr;
+    float sq = 0.f;
+    if (nb + 32 <= N && ((reinterpret_cast<uintptr_t>(wp) & 15u) == 0) &&
+        (!gp || ((reinterpret_cast<uintptr_t>(gp) & 15u) == 0))) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            float4 g, wv = *reinterpret_cast<const float4*>(wp + 4 * q);
+            g.x = u2f(r[4 * q + 0]) * inv_k;
+            g.y = u2f(r[4 * q + 1]) * inv_k;
+            g.z = u2f(r[4 * q + 2]) * inv_k;
+            g.w = u2f(r[4 * q + 3]) * inv_k;
+            wv.x = fmaf(-e.lr, g.x, wv.x);
+            wv.y = fmaf(-e.lr, g.y, wv.y);
+            wv.z = fmaf(-e.lr, g.z, wv.z);
+            wv.w = fmaf(-e.lr, g.w, wv.w);
+            *reinterpret_cast<float4*>(wp + 4 * q) = wv;
+            if (gp) *reinterpret_cast<float4*>(gp + 4 * q) = g;
+            sq += g.x * g.x + g.y * g.y + g.z * g.z + g.w * g.w;
+        }
+    } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            if (nb + j < N) {
+                const float g = u2f(r[j]) * inv_k;
+                wp[j] = fmaf(-e.lr, g, wp[j]);
+                if (gp) gp[j] = g;
+                sq += g * g;
+            }
+        }
+    }
+    return sq;
 }
 
 // ------------------------------------------------------------------ kernel
@@ -377,9 +300,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int mt_n = (M + BM - 1) / BM, nt_n = (N + BN - 1) / BN;
-    const long long total = static_cast<long long>(mt_n) * nt_n;
-    const int nk = (K + BK - 1) / BK;
+    // live extent: rows past (*kdev) * kmul of the row dimension are not computed
+    int Meff = M, Keff = K, live_k = 1;
+    if (epi.kdev) {
+        live_k = *epi.kdev;
+        const long long r = static_cast<long long>(live_k > 0 ? live_k : 0) * epi.kmul;
+        if (KIND == TC_GBAR)
+            Keff = r < K ? static_cast<int>(r) : K;
+        else
+            Meff = r < M ? static_cast<int>(r) : M;
+    }
+    const int mt_n = (Meff + BM - 1) / BM, nt_n = (N + BN - 1) / BN;
+    const long long total = live_k > 0 && Keff > 0 ? static_cast<long long>(mt_n) * nt_n : 0;
+    const int nk = (Keff + BK - 1) / BK;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -480,13 +413,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int m0 = static_cast<int>(t / nt_n) * BM, n0 = static_cast<int>(t % nt_n) * BN;
             const int row = m0 + q * 32 + lane;
             const uint32_t tbase = tmem + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
+            double sq = 0.0;
 #pragma unroll 1
             for (int c = 0; c < BN / 32; ++c) {
                 if (n0 + c * 32 >= N) break;
                 uint32_t r[32];
                 tc_ld_32cols(tbase + c * 32, r);
                 tc_wait_ld();
-                epilogue_chunk<KIND>(epi, 0, row, n0 + c * 32, M, N, r);
+                if constexpr (KIND == TC_GBAR)
+                    sq += gbar_chunk(epi, row, n0 + c * 32, M, N, 1.0f / static_cast<float>(live_k), r);
+                else
+                    epilogue_chunk<KIND>(epi, 0, row, n0 + c * 32, M, N, r);
+            }
+            if constexpr (KIND == TC_GBAR) {
+                // fixed-shape warp tree: the piece of (tile, quarter) does not depend on scheduling
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+                if (lane == 0) epi.pieces[t * 4 + q] = sq;
             }
             tc_fence_before();
             __syncwarp();
@@ -708,38 +651,6 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
 }
 
 // ------------------------------------------------------------------ host side
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn() {
-    static EncodeTiledFn fn = nullptr;
-    static std::once_flag once;
-    std::call_once(once, [] {
-        void* p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(p);
-    });
-    return fn;
-}
-
-// 2-D tensor map of a row-major bf16 matrix [rows, cols] with row stride ld (elements).
-bool make_map(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_k, int box_rows) {
-    EncodeTiledFn fn = encode_fn();
-    if (!fn) return false;
-    cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
-    cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld * 2)};
-    cuuint32_t box[2] = {static_cast<cuuint32_t>(box_k), static_cast<cuuint32_t>(box_rows)};
-    cuuint32_t estr[2] = {1, 1};
-    const CUtensorMapSwizzle sw = box_k == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
-    return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 template <int BK, int STAGES>
 cudaError_t launch_dw(const CUtensorMap& a, const CUtensorMap& b, int Mr, int Nr, int K, int batch, int* status,
                       float* gbase, int64_t ldrow, int64_t ldG, cudaStream_t st) {
@@ -785,6 +696,38 @@ cudaError_t launch_cfg(const CUtensorMap& a, const CUtensorMap& b, int M, int N,
 
 }  // namespace
 
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// 2-D tensor map of a row-major bf16 matrix [rows, cols] with row stride ld (elements).
+bool tc_make_map(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_k, int box_rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld * 2)};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(box_k), static_cast<cuuint32_t>(box_rows)};
+    cuuint32_t estr[2] = {1, 1};
+    const CUtensorMapSwizzle sw = box_k == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+    return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool tc_shape_ok(int64_t lda, int64_t ldb, int K, int64_t kz, const void* A, const void* B) {
     if (!encode_fn()) return false;
     if ((lda % 8) || (ldb % 8) || (kz % 8)) return false;
@@ -805,13 +748,13 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
         // algorithmic bytes: G written once (fp32), both bf16 operands read once
         const double dw_bytes = 4.0 * batch * double(M) * N + 2.0 * batch * double(K) * (double(M) + N);
         void* prof = dw_profile_begin(st, dw_bytes);
-        if (!make_map(&ta, A, rowsA, colsA, lda, bk, BM) || !make_map(&tb, B, rowsB, colsB, ldb, bk, DW_BN))
+        if (!tc_make_map(&ta, A, rowsA, colsA, lda, bk, BM) || !tc_make_map(&tb, B, rowsB, colsB, ldb, bk, DW_BN))
             return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
         float* gb = epi.G + epi.off;
         const bool vec_ok = ((reinterpret_cast<uintptr_t>(gb) & 15u) == 0) && epi.ldrow % 4 == 0 && epi.ldG % 4 == 0;
         if (!vec_ok) {
             // unaligned rows: the one-CTA-per-tile kernel (128-column tiles) with scalar stores
-            if (!make_map(&tb, B, rowsB, colsB, ldb, bk, 128))
+            if (!tc_make_map(&tb, B, rowsB, colsB, ldb, bk, 128))
                 return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
             e = bk == 64 ? launch_cfg<128, 64, 2, TC_DW, 4>(ta, tb, M, N, K, batch, kz, epi, status, st, 48 * 1024)
                          : launch_cfg<128, 32, 2, TC_DW, 4>(ta, tb, M, N, K, batch, kz, epi, status, st, 48 * 1024);
@@ -821,13 +764,15 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
         }
         dw_profile_end(prof, st);
     } else {
-        if (!make_map(&ta, A, rowsA, colsA, lda, 64, BM) || !make_map(&tb, B, rowsB, colsB, ldb, 64, 256))
+        if (!tc_make_map(&ta, A, rowsA, colsA, lda, 64, BM) || !tc_make_map(&tb, B, rowsB, colsB, ldb, 64, 256))
             return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
         // persistent: one CTA per SM (4 stages x 48 KB), 2 x 256 TMEM columns
         if (kind == TC_HIDDEN)
             e = launch_persistent<TC_HIDDEN>(ta, tb, M, N, K, epi, status, st);
         else if (kind == TC_LOGITS)
             e = launch_persistent<TC_LOGITS>(ta, tb, M, N, K, epi, status, st);
+        else if (kind == TC_GBAR)
+            e = launch_persistent<TC_GBAR>(ta, tb, M, N, K, epi, status, st);
         else
             e = launch_persistent<TC_DX>(ta, tb, M, N, K, epi, status, st);
     }

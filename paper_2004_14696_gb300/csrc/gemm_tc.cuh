@@ -2,6 +2,7 @@
 // worker-gradient pass.  Internal interface.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
 
@@ -9,7 +10,7 @@
 
 namespace dbw {
 
-enum TcEpiKind { TC_HIDDEN = 0, TC_LOGITS = 1, TC_DX = 2, TC_DW = 3 };
+enum TcEpiKind { TC_HIDDEN = 0, TC_LOGITS = 1, TC_DX = 2, TC_DW = 3, TC_GBAR = 4 };
 
 // What the epilogue does with accumulator element (m, n) of batch z.
 struct TcEpi {
@@ -24,6 +25,18 @@ struct TcEpi {
     int64_t ldact;
     float* G;                     // DW: G[z * ldG + off + m * ldrow + n] (fp32)
     int64_t ldG, off, ldrow;
+    // GBAR (mean over the received workers, Eqs. (3)-(4)): with g = acc / k,
+    // W[off + m * ldrow + n] -= lr * g, gbar[off + m * ldrow + n] = g (nullable), and the
+    // tile's sum of g^2 (fp64) into pieces[tile * 4 + q] for TMEM lane quarter q.
+    float* W;
+    float* gbar;
+    float lr;
+    double* pieces;
+    // Live row count on the device: when non-null, only (*kdev) * kmul rows of the
+    // row dimension are computed (M for HIDDEN / LOGITS / DX, K for GBAR, where k =
+    // *kdev); *kdev <= 0 runs no tile.
+    const int* kdev;
+    int kmul;
 };
 
 // C[M, N] = sum_{k < K} A[m, z*kz + k] * B[n, z*kz + k] for z < batch, then the
@@ -36,7 +49,25 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
             int64_t ldb, int64_t rowsB, int64_t colsB, int M, int N, int K, int batch, int64_t kz, const TcEpi& epi,
             int* status, cudaStream_t st);
 
+// 2-D TMA tensor map of a row-major bf16 matrix [rows, cols] with row stride ld
+// (elements), box box_k x box_rows, 128-byte (box_k = 64) or 64-byte (32) swizzle;
+// reads past the extents are zero.  False if the driver's encoder is unavailable
+// or rejects the arguments.
+bool tc_make_map(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_k, int box_rows);
+
 // True when tc_gemm can run this problem (alignment rules above).
 bool tc_shape_ok(int64_t lda, int64_t ldb, int K, int64_t kz, const void* A, const void* B);
+
+// Per-worker squared gradient norms of one layer without forming the gradient
+// (the Gram identity ||D^T A||_F^2 = <D D^T, A A^T>_F, with the bias term
+// ||1^T D||^2 = sum of D D^T added):
+//   pieces[(r / 32) * CT + ct] = sum over rows r..r+31 of the 32-row group and the
+//   columns c of the same worker (in column tile ct, CT = max(1, B / 128)) of
+//   (D D^T)[r, c] * ((A A^T)[r, c] + 1)
+// for the row groups of the first (*kdev) * B rows.  A = act [rows, ldA] (K = colsA),
+// D = dz [rows, ldD] (K = colsD), both bf16 row-major; B % 32 == 0 and either
+// 128 % B == 0 or B % 128 == 0.
+int tc_gram(const __nv_bfloat16* act, int64_t ldA, int64_t colsA, const __nv_bfloat16* dz, int64_t ldD,
+            int64_t colsD, int rows, int B, const int* kdev, double* pieces, int* status, cudaStream_t st);
 
 }  // namespace dbw

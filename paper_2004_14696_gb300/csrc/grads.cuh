@@ -49,6 +49,31 @@ struct TcPlan {
     size_t ws_bytes;
 };
 
+// Workspace of the received-workers pass (dbw_received_grads_update): the bf16
+// plan above (its buffers hold the k received workers' rows, slot s = the s-th
+// received worker in increasing index order, at rows s B .. s B + B - 1), then:
+struct RxPlan {
+    TcPlan t;
+    int CT;                            // Gram column tiles per 128-row tile: max(1, B / 128)
+    size_t off_sel;                    // int32 [n]: received workers, increasing
+    size_t off_k;                      // int32: k
+    size_t off_csum;                   // fp32 [n, max out]: per-slot bias gradient sums
+    size_t off_pw[DBW_LMAX];           // fp64 [tiles_l * 4]: pieces of ||g_t(W_l)||^2
+    int64_t npw[DBW_LMAX];
+    size_t off_pb[DBW_LMAX];           // fp64 [ceil(out_l / 128)]: pieces of ||g_t(b_l)||^2
+    int npb[DBW_LMAX];
+    size_t off_pg[DBW_LMAX];           // fp64 [(M / 32) * CT]: Gram pieces of ||g_j||^2
+    size_t ws_bytes;
+};
+
+// The received-workers pass needs the tcgen05 path and a Gram tile layout: B % 32 == 0
+// and either 128 % B == 0 or B % 128 == 0.
+bool rx_eligible(int prec, int B);
+bool make_rx_plan(int L, const int32_t* widths, int n, int B, RxPlan* P);
+int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, const int32_t* labels,
+                      const int32_t* idx, const uint8_t* mask, float lr, float* gbar, float* loss, double* partials,
+                      char* ws, cudaStream_t st);
+
 // The bf16 pass runs on tcgen05 when each worker's sample count is whole 32-deep K blocks.
 bool tc_eligible(int prec, int B);
 bool make_tc_plan(int L, const int32_t* widths, int n, int B, TcPlan* P);

@@ -48,11 +48,24 @@ __global__ void cast_transpose_kernel(const float* __restrict__ W, int out, int 
     }
 }
 
-// dst [cols, ldd] = src [rows, lds]^T  (bf16), rows x cols logical.
+// Rows of the stacked buffers that a received-workers pass computes: the k B
+// received rows rounded up to the 128-row GEMM tile (all M when kdev is null).
+__device__ __forceinline__ int live_rows(const int* kdev, int B, int M) {
+    if (!kdev) return M;
+    const int k = *kdev;
+    const long long r = (static_cast<long long>(k > 0 ? k : 0) * B + 127) / 128 * 128;
+    return r < M ? static_cast<int>(r) : M;
+}
+
+// dst [cols, ldd] = src [rows, lds]^T  (bf16), rows x cols logical; with kdev, only
+// the live rows (live_rows) are transposed.
 __global__ void transpose_bf16_kernel(const __nv_bfloat16* __restrict__ src, int rows, int cols, int64_t lds,
-                                      __nv_bfloat16* __restrict__ dst, int64_t ldd) {
+                                      __nv_bfloat16* __restrict__ dst, int64_t ldd, const int* kdev = nullptr,
+                                      int B = 0) {
     __shared__ __nv_bfloat16 tile[32][33];
     const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+    rows = live_rows(kdev, B, rows);
+    if (r0 >= rows) return;
     const int tx = threadIdx.x, ty = threadIdx.y;
     for (int r = ty; r < 32; r += 8) {
         const int rr = r0 + r, cc = c0 + tx;
@@ -89,21 +102,37 @@ __global__ void gather_bf16_kernel(const float* __restrict__ pool, int64_t S, in
 
 // Per worker (one CTA): stable log-softmax cross entropy per sample, dZ = (softmax - onehot) / B
 // as bf16 into dZ [M, ldz], worker loss = mean of its B sample losses (sample order).
+// With ``sel`` (received-workers pass): CTA s handles slot s, i.e. worker sel[s]
+// (stacked rows s B .., samples idx[sel[s] B + r], loss[sel[s]]); slots s >= k
+// zero their dZ rows up to the live row count and stop.
 __global__ void __launch_bounds__(256) softmax_xent_ld_kernel(const float* __restrict__ logits, int64_t ldl, int C,
                                                               int B, const int32_t* __restrict__ idx, int64_t S,
                                                               const int32_t* __restrict__ labels,
                                                               float* __restrict__ sample_loss,
                                                               __nv_bfloat16* __restrict__ dZ, int64_t ldz,
-                                                              float* __restrict__ loss) {
+                                                              float* __restrict__ loss,
+                                                              const int32_t* __restrict__ sel = nullptr,
+                                                              const int* __restrict__ kdev = nullptr) {
     const int i = blockIdx.x;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    int worker = i;
+    if (sel) {
+        if (i >= *kdev) {
+            const int live = live_rows(kdev, B, gridDim.x * B);
+            for (int r = warp; r < B && i * B + r < live; r += nw)
+                for (int c = lane; c < C; c += 32)
+                    dZ[(static_cast<int64_t>(i) * B + r) * ldz + c] = __float2bfloat16_rn(0.f);
+            return;
+        }
+        worker = sel[i];
+    }
     __shared__ int bad_s;
     if (threadIdx.x == 0) bad_s = 0;
     __syncthreads();
     const float invB = 1.0f / static_cast<float>(B);
     for (int r = warp; r < B; r += nw) {
         const int64_t row = static_cast<int64_t>(i) * B + r;
-        const int64_t sidx = idx[row];
+        const int64_t sidx = idx[static_cast<int64_t>(worker) * B + r];
         int y = -1;
         if (sidx >= 0 && sidx < S) y = labels[sidx];
         const bool bad = (y < 0 || y >= C);
@@ -131,7 +160,7 @@ __global__ void __launch_bounds__(256) softmax_xent_ld_kernel(const float* __res
     if (threadIdx.x == 0) {
         float acc = 0.f;
         for (int r = 0; r < B; ++r) acc += sample_loss[static_cast<int64_t>(i) * B + r];
-        loss[i] = bad_s ? NAN : acc * invB;
+        loss[worker] = bad_s ? NAN : acc * invB;
     }
 }
 
@@ -145,6 +174,170 @@ __global__ void bias_grad_ld_kernel(const __nv_bfloat16* __restrict__ dZ, int64_
     float acc = 0.f;
     for (int r = 0; r < B; ++r) acc += __bfloat162float(p[static_cast<int64_t>(r) * ldz]);
     G[static_cast<int64_t>(i) * ldG + offb + o] = acc;
+}
+
+// ------------------------------------------------------------------ received-workers pass
+// sel[0..k) = the workers with mask[j] != 0 in increasing order, *kout = k, and
+// loss[j] = NaN for the others (their gradients are never formed).  One CTA of
+// 1024 threads: a ballot prefix count per warp, then over the warp totals.
+__global__ void __launch_bounds__(1024) compact_received_kernel(const uint8_t* __restrict__ mask, int n,
+                                                                int32_t* __restrict__ sel, int* __restrict__ kout,
+                                                                float* __restrict__ loss) {
+    __shared__ int warp_tot[32];
+    const int j = threadIdx.x, lane = j & 31, warp = j >> 5;
+    const bool on = j < n && mask[j] != 0;
+    const unsigned bal = __ballot_sync(0xffffffffu, on);
+    if (lane == 0) warp_tot[warp] = __popc(bal);
+    __syncthreads();
+    int base = 0;
+    for (int q = 0; q < warp; ++q) base += warp_tot[q];
+    if (on) sel[base + __popc(bal & ((1u << lane) - 1u))] = j;
+    else if (j < n) loss[j] = NAN;
+    if (j == 0) {
+        int k = 0;
+        for (int q = 0; q < 32; ++q) k += warp_tot[q];
+        *kout = k;
+    }
+}
+
+// X[m, :] = bf16(pool[idx[sel[s] B + r], :]) for m = s B + r, s < k; live rows past
+// k B are zeroed (so every stacked row a GEMM tile reads is finite).
+__global__ void gather_received_kernel(const float* __restrict__ pool, int64_t S, int in,
+                                       const int32_t* __restrict__ idx, const int32_t* __restrict__ sel,
+                                       const int* __restrict__ kdev, int B, int M, __nv_bfloat16* __restrict__ X,
+                                       int64_t ldx) {
+    const int k = *kdev;
+    const int live = live_rows(kdev, B, M);
+    for (int m = blockIdx.y; m < live; m += gridDim.y) {
+        const int s = m / B;
+        __nv_bfloat16* dst = X + static_cast<int64_t>(m) * ldx;
+        if (s >= k) {
+            for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < in; c += gridDim.x * blockDim.x)
+                dst[c] = __float2bfloat16_rn(0.f);
+            continue;
+        }
+        int64_t r = idx[static_cast<int64_t>(sel[s]) * B + (m - s * B)];
+        if (r < 0 || r >= S) r = 0;   // the loss kernel poisons that worker
+        const float* src = pool + r * in;
+        for (int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4; c < in; c += gridDim.x * blockDim.x * 4) {
+            const float4 v = *reinterpret_cast<const float4*>(src + c);
+            if (c + 3 < in) {
+                *reinterpret_cast<__nv_bfloat162*>(dst + c) = __floats2bfloat162_rn(v.x, v.y);
+                *reinterpret_cast<__nv_bfloat162*>(dst + c + 2) = __floats2bfloat162_rn(v.z, v.w);
+            } else {
+                for (int e = c; e < in; ++e) dst[e] = __float2bfloat16_rn(src[e]);
+            }
+        }
+    }
+}
+
+// csum[s * out + o] = sum_{r < B} dZ[s B + r, o] (rows in order) for slots s < k:
+// worker sel[s]'s bias gradient, the same sums the per-worker pass writes into G.
+__global__ void slot_colsum_kernel(const __nv_bfloat16* __restrict__ dZ, int64_t ldz, int out, int B,
+                                   const int* __restrict__ kdev, float* __restrict__ csum) {
+    const int s = blockIdx.y;
+    const int o = blockIdx.x * blockDim.x + threadIdx.x;
+    if (s >= *kdev || o >= out) return;
+    const __nv_bfloat16* p = dZ + static_cast<int64_t>(s) * B * ldz + o;
+    float acc = 0.f;
+    for (int r = 0; r < B; ++r) acc += __bfloat162float(p[static_cast<int64_t>(r) * ldz]);
+    csum[static_cast<int64_t>(s) * out + o] = acc;
+}
+
+// Bias part of Eqs. (3)-(4): g = (1/k) sum_{s < k} csum[s, o] (slots in order),
+// wb[o] -= lr g, gb[o] = g (nullable); the CTA's sum of g^2 (fp64, fixed tree)
+// into pieces[blockIdx.x].
+__global__ void __launch_bounds__(128) bias_mean_update_kernel(const float* __restrict__ csum, int out,
+                                                               const int* __restrict__ kdev, float lr,
+                                                               float* __restrict__ wb, float* __restrict__ gb,
+                                                               double* __restrict__ pieces) {
+    __shared__ double red[128];
+    const int k = *kdev;
+    const int o = blockIdx.x * blockDim.x + threadIdx.x;
+    double sq = 0.0;
+    if (o < out && k > 0) {
+        float acc = 0.f;
+        for (int s = 0; s < k; ++s) acc += csum[static_cast<int64_t>(s) * out + o];
+        const float g = acc * (1.0f / static_cast<float>(k));
+        wb[o] = fmaf(-lr, g, wb[o]);
+        if (gb) gb[o] = g;
+        sq = static_cast<double>(g) * g;
+    }
+    red[threadIdx.x] = sq;
+    __syncthreads();
+    for (int h = 64; h > 0; h >>= 1) {
+        if (threadIdx.x < h) red[threadIdx.x] += red[threadIdx.x + h];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) pieces[blockIdx.x] = red[0];
+}
+
+struct FinishArgs {
+    int L, n, B, CT;
+    const double* pw[DBW_LMAX];   // tile pieces of ||g_t(W_l)||^2
+    int64_t npw[DBW_LMAX];
+    const double* pb[DBW_LMAX];   // CTA pieces of ||g_t(b_l)||^2
+    int npb[DBW_LMAX];
+    const double* pg[DBW_LMAX];   // Gram pieces, [(row group) * CT + ct]
+};
+
+// Writes the partials buffer dbw_grad_stats reads (one block per quantity):
+//   vals[j] = ||g_j||^2 for received j (sum over layers and the worker's Gram pieces),
+//             0 for the others;
+//   vals[n + 1] = ||g_t||^2 (all W and b pieces);
+//   vals[n] = sum_j ||g_j||^2 - k ||g_t||^2, the deviation sum of Eq. (10) by the
+//             identity sum_j ||g_j - g_t||^2 = sum_j ||g_j||^2 - k ||g_t||^2 (fp64).
+// Every sum runs in a fixed order (strided per thread, then a fixed tree).
+__global__ void __launch_bounds__(256) finish_received_kernel(FinishArgs a, const int32_t* __restrict__ sel,
+                                                              const int* __restrict__ kdev,
+                                                              double* __restrict__ partials) {
+    __shared__ double red[2][256];
+    const int t = threadIdx.x, n = a.n;
+    const int k = *kdev;
+    int64_t* hdr = reinterpret_cast<int64_t*>(partials);
+    double* vals = partials + kPartialsHeader + (n + 2);
+    if (t == 0) {
+        hdr[0] = kPartialsMagic;
+        hdr[1] = 1;
+        hdr[2] = n;
+        hdr[3] = 0;
+    }
+    for (int j = t; j < n; j += 256) vals[j] = 0.0;
+    double g2 = 0.0, rs = 0.0;
+    for (int l = 0; l < a.L; ++l) {
+        for (int64_t i = t; i < a.npw[l]; i += 256) g2 += a.pw[l][i];
+        for (int i = t; i < a.npb[l]; i += 256) g2 += a.pb[l][i];
+    }
+    __syncthreads();   // zeros above land before the received rows below
+    const int groups = a.B / 32;   // 32-row groups per worker
+    for (int s = t; s < k; s += 256) {
+        double v = 0.0;
+        for (int l = 0; l < a.L; ++l) {
+            const double* pg = a.pg[l] + static_cast<int64_t>(s) * groups * a.CT;
+            for (int i = 0; i < groups * a.CT; ++i) v += pg[i];
+        }
+        vals[sel[s]] = v;
+        rs += v;
+    }
+    red[0][t] = g2;
+    red[1][t] = rs;
+    __syncthreads();
+    for (int h = 128; h > 0; h >>= 1) {
+        if (t < h) {
+            red[0][t] += red[0][t + h];
+            red[1][t] += red[1][t + h];
+        }
+        __syncthreads();
+    }
+    if (t == 0) {
+        if (k > 0) {
+            vals[n + 1] = red[0][0];
+            vals[n] = red[1][0] - static_cast<double>(k) * red[0][0];
+        } else {
+            vals[n + 1] = NAN;
+            vals[n] = NAN;
+        }
+    }
 }
 
 }  // namespace
@@ -282,6 +475,193 @@ int worker_grads_tc(const TcPlan& P, const float* w, const float* pool, int64_t 
         }
     }
     return DBW_OK;
+}
+
+// ------------------------------------------------------------------ received-workers pass
+// Eqs. (2)-(4) and the statistics of Sect. 3.1 for the k received workers only,
+// without the [n, d] gradient matrix: the rows of the received workers are
+// stacked (slot s = s-th received worker), the forward and input-gradient GEMMs
+// run over those k B rows, the weight part of g_t is one GEMM with K = k B whose
+// epilogue applies the SGD step (TC_GBAR), the bias part is a column sum, and the
+// per-worker squared norms come from B x B Gram matrices (tc_gram).  The number
+// of received workers k is read on the device from ``mask``.
+
+bool rx_eligible(int prec, int B) { return tc_eligible(prec, B) && (128 % B == 0 || B % 128 == 0); }
+
+bool make_rx_plan(int L, const int32_t* widths, int n, int B, RxPlan* P) {
+    if (!make_tc_plan(L, widths, n, B, &P->t)) return false;
+    const GradsPlan& g = P->t.g;
+    P->CT = B > 128 ? B / 128 : 1;
+    size_t cur = P->t.ws_bytes;
+    auto take = [&](size_t bytes) {
+        const size_t at = cur;
+        cur += (bytes + 255) / 256 * 256;
+        return at;
+    };
+    int maxout = 0;
+    for (int l = 0; l < L; ++l) maxout = g.widths[l + 1] > maxout ? g.widths[l + 1] : maxout;
+    P->off_sel = take(static_cast<size_t>(n) * 4);
+    P->off_k = take(4);
+    P->off_csum = take(static_cast<size_t>(n) * maxout * 4);
+    for (int l = 0; l < L; ++l) {
+        const int fin = g.widths[l], fout = g.widths[l + 1];
+        P->npw[l] = static_cast<int64_t>((fout + 127) / 128) * ((fin + 255) / 256) * 4;
+        P->off_pw[l] = take(static_cast<size_t>(P->npw[l]) * 8);
+        P->npb[l] = (fout + 127) / 128;
+        P->off_pb[l] = take(static_cast<size_t>(P->npb[l]) * 8);
+        P->off_pg[l] = take(static_cast<size_t>(g.M / 32) * P->CT * 8);
+    }
+    P->ws_bytes = cur;
+    return true;
+}
+
+int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, const int32_t* labels,
+                      const int32_t* idx, const uint8_t* mask, float lr, float* gbar, float* loss, double* partials,
+                      char* ws, cudaStream_t st) {
+    const TcPlan& T = P.t;
+    const GradsPlan& g = T.g;
+    const int L = g.L, M = g.M, B = g.B, n = g.n;
+    int* status = reinterpret_cast<int*>(ws + T.off_status);
+    int32_t* sel = reinterpret_cast<int32_t*>(ws + P.off_sel);
+    int* kdev = reinterpret_cast<int*>(ws + P.off_k);
+    float* csum = reinterpret_cast<float*>(ws + P.off_csum);
+    auto bf = [&](size_t off) { return reinterpret_cast<__nv_bfloat16*>(ws + off); };
+    auto f64 = [&](size_t off) { return reinterpret_cast<double*>(ws + off); };
+    const char* what = "dbw_received_grads_update";
+    cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int), st);
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+
+    compact_received_kernel<<<1, 1024, 0, st>>>(mask, n, sel, kdev, loss);
+    for (int l = 0; l < L; ++l) {
+        const int fin = g.widths[l], fout = g.widths[l + 1];
+        dim3 grid((fin + 31) / 32, (fout + 31) / 32);
+        cast_transpose_kernel<<<grid, dim3(32, 8), 0, st>>>(w + g.offW[l], fout, fin, bf(T.off_wb[l]), T.ldw[l],
+                                                            bf(T.off_wt[l]), T.ldwt[l]);
+    }
+    {
+        const int in = g.widths[0];
+        dim3 grid((in + 1023) / 1024, M < 65535 ? M : 65535);
+        gather_received_kernel<<<grid, 256, 0, st>>>(pool, S, in, idx, sel, kdev, B, M, bf(T.off_act[0]), T.ldact[0]);
+        dim3 tg((in + 31) / 32, (M + 31) / 32);
+        transpose_bf16_kernel<<<tg, dim3(32, 8), 0, st>>>(bf(T.off_act[0]), M, in, T.ldact[0], bf(T.off_actT[0]),
+                                                          T.M8, kdev, B);
+    }
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+
+    // forward over the live rows
+    float* logits = reinterpret_cast<float*>(ws + T.off_logits);
+    for (int l = 0; l < L; ++l) {
+        const int fin = g.widths[l], fout = g.widths[l + 1];
+        TcEpi ep{};
+        ep.bias = w + g.offb[l];
+        ep.kdev = kdev;
+        ep.kmul = B;
+        int rc;
+        if (l < L - 1) {
+            ep.out = bf(T.off_act[l + 1]);
+            ep.ldo = T.ldact[l + 1];
+            ep.outT = bf(T.off_actT[l + 1]);
+            ep.ldT = T.M8;
+            rc = tc_gemm(TC_HIDDEN, bf(T.off_act[l]), T.ldact[l], M, fin, bf(T.off_wb[l]), T.ldw[l], fout, fin, M,
+                         fout, fin, 1, 0, ep, status, st);
+        } else {
+            ep.outF = logits;
+            ep.ldF = T.ldlog;
+            rc = tc_gemm(TC_LOGITS, bf(T.off_act[l]), T.ldact[l], M, fin, bf(T.off_wb[l]), T.ldw[l], fout, fin, M,
+                         fout, fin, 1, 0, ep, status, st);
+        }
+        if (rc) return rc;
+    }
+    const int C = g.widths[L];
+    float* sloss = reinterpret_cast<float*>(ws + T.off_sloss);
+    int cur = 0;
+    softmax_xent_ld_kernel<<<n, 256, 0, st>>>(logits, T.ldlog, C, B, idx, S, labels, sloss, bf(T.off_dz[0]), T.ldz,
+                                              loss, sel, kdev);
+    {
+        dim3 tg((C + 31) / 32, (M + 31) / 32);
+        transpose_bf16_kernel<<<tg, dim3(32, 8), 0, st>>>(bf(T.off_dz[0]), M, C, T.ldz, bf(T.off_dzT), T.M8, kdev,
+                                                          B);
+    }
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+
+    // backward: mean gradient + SGD step, bias, Gram norms, then dZ of the layer below
+    for (int l = L - 1; l >= 0; --l) {
+        const int fin = g.widths[l], fout = g.widths[l + 1];
+        TcEpi gb{};
+        gb.W = w;
+        gb.gbar = gbar;
+        gb.lr = lr;
+        gb.off = g.offW[l];
+        gb.ldrow = fin;
+        gb.pieces = f64(P.off_pw[l]);
+        gb.kdev = kdev;
+        gb.kmul = B;
+        int rc = tc_gemm(TC_GBAR, bf(T.off_dzT), T.M8, fout, M, bf(T.off_actT[l]), T.M8, fin, M, fout, fin, M, 1, 0,
+                         gb, status, st);
+        if (rc) return rc;
+        slot_colsum_kernel<<<dim3((fout + 127) / 128, n), 128, 0, st>>>(bf(T.off_dz[cur]), T.ldz, fout, B, kdev,
+                                                                         csum);
+        bias_mean_update_kernel<<<P.npb[l], 128, 0, st>>>(csum, fout, kdev, lr, w + g.offb[l],
+                                                           gbar ? gbar + g.offb[l] : nullptr, f64(P.off_pb[l]));
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+        rc = tc_gram(bf(T.off_act[l]), T.ldact[l], fin, bf(T.off_dz[cur]), T.ldz, fout, M, B, kdev, f64(P.off_pg[l]),
+                     status, st);
+        if (rc) return rc;
+        if (l > 0) {
+            TcEpi ex{};
+            ex.act = bf(T.off_act[l]);
+            ex.ldact = T.ldact[l];
+            ex.out = bf(T.off_dz[cur ^ 1]);
+            ex.ldo = T.ldz;
+            ex.outT = bf(T.off_dzT);
+            ex.ldT = T.M8;
+            ex.kdev = kdev;
+            ex.kmul = B;
+            rc = tc_gemm(TC_DX, bf(T.off_dz[cur]), T.ldz, M, fout, bf(T.off_wt[l]), T.ldwt[l], fin, fout, M, fin,
+                         fout, 1, 0, ex, status, st);
+            if (rc) return rc;
+            cur ^= 1;
+        }
+    }
+    FinishArgs fa{};
+    fa.L = L;
+    fa.n = n;
+    fa.B = B;
+    fa.CT = P.CT;
+    for (int l = 0; l < L; ++l) {
+        fa.pw[l] = f64(P.off_pw[l]);
+        fa.npw[l] = P.npw[l];
+        fa.pb[l] = f64(P.off_pb[l]);
+        fa.npb[l] = P.npb[l];
+        fa.pg[l] = f64(P.off_pg[l]);
+    }
+    finish_received_kernel<<<1, 256, 0, st>>>(fa, sel, kdev, partials);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+    return DBW_OK;
+}
+
+size_t received_workspace_bytes(int L, const int32_t* widths, int n, int B, int prec) {
+    RxPlan P;
+    if (!rx_eligible(prec, B) || !make_rx_plan(L, widths, n, B, &P)) return 0;
+    return P.ws_bytes;
+}
+
+int launch_received_grads(int L, const int32_t* widths, int prec, float* w, int64_t d, const float* pool, int64_t S,
+                          const int32_t* labels, const int32_t* idx, int n, int B, const uint8_t* mask, float lr,
+                          float* gbar, float* loss, double* partials, void* ws, size_t ws_bytes, cudaStream_t st) {
+    const char* what = "dbw_received_grads_update";
+    if (!rx_eligible(prec, B))
+        return fail(DBW_EUNSUPPORTED, "%s: needs prec = DBW_PREC_BF16, B %% 32 == 0 and B | 128 or 128 | B", what);
+    RxPlan P;
+    if (!make_rx_plan(L, widths, n, B, &P)) return fail(DBW_EINVAL, "%s: invalid model shape", what);
+    if (d != P.t.g.d) return fail(DBW_EINVAL, "%s: d = %lld, the widths give %lld", what, (long long)d,
+                                  (long long)P.t.g.d);
+    if (ws_bytes < P.ws_bytes) return fail(DBW_EINVAL, "%s: workspace %zu bytes < %zu needed", what, ws_bytes, P.ws_bytes);
+    return received_grads_tc(P, w, pool, S, labels, idx, mask, lr, gbar, loss, partials, static_cast<char*>(ws), st);
 }
 
 }  // namespace dbw

@@ -63,6 +63,10 @@ _SIGS = {
     "dbw_aggregate_partials_bytes": (_sz, [_i32, _i64]),
     "dbw_aggregate_update": (_i32, [_vp, _i64, _i32, _i64, _vp, _f32, _vp, _vp, _vp, _sz, _vp]),
     "dbw_aggregate_update_noalloc": (_i32, [_vp, _i64, _i32, _i64, _vp, _f32, _vp, _vp, _vp, _vp]),
+    "dbw_received_grads_workspace_bytes": (_sz, [_i32, _vp, _i32, _i32, _i32]),
+    "dbw_received_partials_bytes": (_sz, [_i32]),
+    "dbw_received_grads_update": (_i32, [_i32, _vp, _i32, _vp, _i64, _vp, _i64, _vp, _vp, _i32, _i32, _vp, _f32,
+                                         _vp, _vp, _vp, _sz, _vp, _sz, _vp]),
     "dbw_state_init": (_i32, [_vp, _i32, _i32, _vp]),
     "dbw_grad_stats": (_i32, [_vp, _i32, _vp, _vp, _vp, _f64, _vp, _vp, _vp, _vp]),
     "dbw_choose_b": (_i32, [_vp, _f64, _f64, _i32, _vp, _vp, _vp]),
@@ -152,6 +156,15 @@ def dbw_aggregate_partials_bytes(n, d):
     return int(lib().dbw_aggregate_partials_bytes(n, d))
 
 
+def dbw_received_grads_workspace_bytes(widths, n, B, prec):
+    L, arr = _widths(widths)
+    return int(lib().dbw_received_grads_workspace_bytes(L, arr, n, B, prec))
+
+
+def dbw_received_partials_bytes(n):
+    return int(lib().dbw_received_partials_bytes(n))
+
+
 # ----------------------------------------------------------------- compute
 def dbw_worker_grads(widths, prec, w, pool, labels, idx, n, B, G, loss, ws, stream=None):
     L, arr = _widths(widths)
@@ -161,6 +174,20 @@ def dbw_worker_grads(widths, prec, w, pool, labels, idx, n, B, G, loss, ws, stre
         _ptr(labels, torch.int32, "labels"), _ptr(idx, torch.int32, "idx"), n, B, _ptr(G, torch.float32, "G"),
         G.shape[1], _ptr(loss, torch.float32, "loss"), _ptr(ws, torch.uint8, "ws"), ws.numel(), _stream(stream))
     _check("dbw_worker_grads", rc)
+
+
+def dbw_received_grads_update(widths, prec, w, pool, labels, idx, n, B, mask, lr, loss, partials, ws, gbar=None,
+                              stream=None):
+    """One iteration for the received workers only (no [n, d] matrix): w updated in
+    place, loss [n] (NaN for workers mask leaves out), partials for dbw_grad_stats."""
+    L, arr = _widths(widths)
+    rc = lib().dbw_received_grads_update(
+        L, arr, prec, _ptr(w, torch.float32, "w"), w.numel(), _ptr(pool, torch.float32, "pool"), pool.shape[0],
+        _ptr(labels, torch.int32, "labels"), _ptr(idx, torch.int32, "idx"), n, B, _ptr(mask, torch.uint8, "mask"),
+        float(lr), _ptr(gbar, torch.float32, "gbar", nullable=True), _ptr(loss, torch.float32, "loss"),
+        _ptr(partials, torch.uint8, "partials"), partials.numel(), _ptr(ws, torch.uint8, "ws"), ws.numel(),
+        _stream(stream))
+    _check("dbw_received_grads_update", rc)
 
 
 def dbw_select_fastest(times, b, order, mask, tsorted, k_out=None, stream=None):

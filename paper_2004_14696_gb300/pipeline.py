@@ -7,6 +7,11 @@ paper's order (Sect. 3: b_t is chosen right after w_t is available):
     dbw_choose_b -> dbw_worker_grads -> dbw_select_fastest
                  -> dbw_aggregate_update -> dbw_grad_stats
 
+or, with ``received=True`` (the same iteration without the [n, d] gradient
+matrix, for the k received workers only):
+
+    dbw_choose_b -> dbw_select_fastest -> dbw_received_grads_update -> dbw_grad_stats
+
 Python only sequences the calls and owns memory through torch; every step of
 the computation runs in libdbw's kernels on the current CUDA stream.
 """
@@ -21,13 +26,14 @@ from .workloads import Workload
 
 class Iteration:
     def __init__(self, wl: Workload, device="cuda", static_b=None, blind=False, keep_gbar=False,
-                 pool=None, labels=None, w0=None):
+                 pool=None, labels=None, w0=None, received=False):
         self.wl = wl
         self.device = torch.device(device)
         n, d, ld = wl.n, wl.d, wl.ld
         self.n, self.d, self.ld = n, d, ld
         self.static_b = static_b
         self.blind = blind
+        self.received = received
         if pool is None:
             pool = inputs.feature_pool(wl.seed, wl.S, wl.widths[0], wl.feature_dist)
         if labels is None:
@@ -37,11 +43,20 @@ class Iteration:
         self.pool = torch.as_tensor(pool).to(self.device)
         self.labels = torch.as_tensor(labels).to(self.device)
         self.w = torch.as_tensor(w0).to(self.device).clone()
-        self.G = torch.empty((n, ld), dtype=torch.float32, device=self.device)
         self.loss = torch.empty(n, dtype=torch.float32, device=self.device)
-        self.ws = torch.empty(dbw.dbw_worker_grads_workspace_bytes(wl.widths, n, wl.B, wl.prec),
-                              dtype=torch.uint8, device=self.device)
-        self.partials = torch.empty(dbw.dbw_aggregate_partials_bytes(n, d), dtype=torch.uint8, device=self.device)
+        if received:
+            wsb = dbw.dbw_received_grads_workspace_bytes(wl.widths, n, wl.B, wl.prec)
+            if wsb == 0:
+                raise ValueError(f"{wl.key}: the received-workers pass needs bf16, B % 32 == 0, B | 128 or 128 | B")
+            self.G = None
+            self.ws = torch.empty(wsb, dtype=torch.uint8, device=self.device)
+            self.partials = torch.empty(dbw.dbw_received_partials_bytes(n), dtype=torch.uint8, device=self.device)
+        else:
+            self.G = torch.empty((n, ld), dtype=torch.float32, device=self.device)
+            self.ws = torch.empty(dbw.dbw_worker_grads_workspace_bytes(wl.widths, n, wl.B, wl.prec),
+                                  dtype=torch.uint8, device=self.device)
+            self.partials = torch.empty(dbw.dbw_aggregate_partials_bytes(n, d), dtype=torch.uint8,
+                                        device=self.device)
         self.state = dbw.new_state(n, wl.D, self.device)
         self.b = torch.zeros(1, dtype=torch.int32, device=self.device)
         if static_b is not None:
@@ -81,10 +96,15 @@ class Iteration:
                              dbw.CHOOSE_BLIND if self.blind else 0, stream)
         # static b is known on the host: its learning-rate rule applies; DBW uses lr
         lr = wl.lr if self.static_b is None else wl.lr_for(wl.n - int(self.static_b))
-        dbw.dbw_worker_grads(wl.widths, wl.prec, self.w, self.pool, self.labels, idx, wl.n, wl.B, self.G,
-                             self.loss, self.ws, stream)
-        dbw.dbw_select_fastest(times, self.b, self.order, self.mask, self.tsorted, self.k, stream)
-        dbw.dbw_aggregate_update(self.G, wl.n, self.d, self.mask, lr, self.w, self.partials, self.gbar, stream)
+        if self.received:
+            dbw.dbw_select_fastest(times, self.b, self.order, self.mask, self.tsorted, self.k, stream)
+            dbw.dbw_received_grads_update(wl.widths, wl.prec, self.w, self.pool, self.labels, idx, wl.n, wl.B,
+                                          self.mask, lr, self.loss, self.partials, self.ws, self.gbar, stream)
+        else:
+            dbw.dbw_worker_grads(wl.widths, wl.prec, self.w, self.pool, self.labels, idx, wl.n, wl.B, self.G,
+                                 self.loss, self.ws, stream)
+            dbw.dbw_select_fastest(times, self.b, self.order, self.mask, self.tsorted, self.k, stream)
+            dbw.dbw_aggregate_update(self.G, wl.n, self.d, self.mask, lr, self.w, self.partials, self.gbar, stream)
         dbw.dbw_grad_stats(self.partials, wl.n, self.mask, self.loss, self.tsorted, lr, self.state, self.stats,
                            self.row_sqnorm, stream)
 
@@ -122,6 +142,12 @@ class Iteration:
     def launches_per_step(self):
         """Kernels libdbw launches per step (for the bench's launch count)."""
         L = len(self.wl.widths) - 1
+        choose = 0 if self.static_b is not None else 1
+        if self.received:
+            # select; status memset, compaction, L weight cast-transposes, gather + X^T, L forward
+            # GEMMs, loss + dZ^T, per layer (mean-gradient GEMM, bias sums, bias update, Gram),
+            # L-1 dX GEMMs, finish; grad_stats (2)
+            return choose + 1 + (1 + 1 + L + 2 + L + 2 + 4 * L + (L - 1) + 1) + 2
         if self.wl.prec == dbw.PREC_BF16 and self.wl.B % 32 == 0:
             # tcgen05 pass: status memset, L weight cast-transposes, gather + X^T, L forward
             # GEMMs, loss + dZ^T, L dW GEMMs, L bias gradients, L-1 dX GEMMs
@@ -130,7 +156,7 @@ class Iteration:
             grads = 1 + 1 + L + 1 + L + L + (L - 1)    # status memset, gather, fwd, loss, dW, bias, dX
             if self.wl.prec == dbw.PREC_BF16:
                 grads += 1                              # bf16 weight cast
-        return (0 if self.static_b is not None else 1) + grads + 1 + 1 + 2
+        return choose + grads + 1 + 1 + 2
 
 
 def agg_case(n, d, seed, b, device="cuda", mean=0.0, std=1.0):
@@ -142,7 +168,8 @@ def agg_case(n, d, seed, b, device="cuda", mean=0.0, std=1.0):
     return G, w, times
 
 
-def run(wl: Workload, iters, log=None, static_b=None, blind=False, device="cuda", start=0, it=None):
+def run(wl: Workload, iters, log=None, static_b=None, blind=False, device="cuda", start=0, it=None,
+        received=False):
     """Run ``iters`` iterations of a workload; returns (and optionally writes as JSON
     lines to the file object ``log``) one record per iteration: b_t, k_t, the k_t-th
     arrival time T_(k_t) (the iteration's virtual duration), the virtual clock, F^_t,
@@ -150,7 +177,7 @@ def run(wl: Workload, iters, log=None, static_b=None, blind=False, device="cuda"
     import json
     import time
     if it is None:
-        it = Iteration(wl, device=device, static_b=static_b, blind=blind)
+        it = Iteration(wl, device=device, static_b=static_b, blind=blind, received=received)
     out = []
     for t in range(start, start + iters):
         it.load_inputs(t)
@@ -173,12 +200,14 @@ def _main(argv=None):
     p.add_argument("--iters", type=int, default=None)
     p.add_argument("--static-b", type=int, default=None)
     p.add_argument("--blind", action="store_true", help="B-DBW: the gain of k is k itself")
+    p.add_argument("--received", action="store_true",
+                   help="received workers only, without the [n, d] gradient matrix")
     p.add_argument("--log", default="-")
     a = p.parse_args(argv)
     wl = workloads.ALL[a.workload]
     f = sys.stdout if a.log == "-" else open(a.log, "w")
     try:
-        run(wl, a.iters or wl.iters, f, a.static_b, a.blind)
+        run(wl, a.iters or wl.iters, f, a.static_b, a.blind, received=a.received)
     finally:
         if f is not sys.stdout:
             f.close()

@@ -3,6 +3,7 @@
     python -m paper_2004_14696_gb300.profile_case aggregate --n 64 --d 4000000 --b 16 --reps 3
     python -m paper_2004_14696_gb300.profile_case sweep            # the aggregation-only sweep
     python -m paper_2004_14696_gb300.profile_case grads --workload mlp4096x3-1000_n256_B32 --reps 3
+    python -m paper_2004_14696_gb300.profile_case received --workload mlp4096x3-1000_n256_B32 --b 64
 
 Each prints one JSON line per case with CUDA-event times (on the launching
 stream, after warm-up).  Large gradient matrices are filled on the device with
@@ -89,6 +90,39 @@ def grads_case(key, reps, warmup=2):
             "TFLOP_s": flop / (avg * 1e-3) / 1e12, "G_write_GB_s": wl.n * wl.ld * 4 / (avg * 1e-3) / 1e9}
 
 
+def received_case(key, b, reps, warmup=2):
+    """dbw_received_grads_update alone (after one selection with static b): the received
+    workers' gradients, mean, SGD step and norms without the [n, d] matrix."""
+    wl = workloads.ALL[key]
+    it = Iteration(wl, static_b=b, received=True)
+    it.load_inputs(0)
+    dbw.dbw_select_fastest(it.times, it.b, it.order, it.mask, it.tsorted, it.k)
+
+    def call():
+        dbw.dbw_received_grads_update(wl.widths, wl.prec, it.w, it.pool, it.labels, it.idx, wl.n, wl.B, it.mask,
+                                      wl.lr, it.loss, it.partials, it.ws)
+    for _ in range(warmup):
+        call()
+    st = torch.cuda.current_stream()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    torch.cuda.synchronize()
+    for e0, e1 in evs:
+        e0.record(st)
+        call()
+        e1.record(st)
+    torch.cuda.synchronize()
+    ms = [e0.elapsed_time(e1) for e0, e1 in evs]
+    k = wl.n - b
+    Mk = k * wl.B
+    flop = 0
+    for l in range(len(wl.widths) - 1):
+        flop += 2 * Mk * wl.widths[l] * wl.widths[l + 1] * (3 if l else 2)
+    avg = float(np.mean(ms))
+    return {"case": "received_update", "workload": key, "b": b, "k": k, "ms": avg, "ms_min": min(ms),
+            "flop": flop, "TFLOP_s": flop / (avg * 1e-3) / 1e12,
+            "status": int(it.ws[:4].view(torch.int32).item())}
+
+
 def main(argv=None):
     p = argparse.ArgumentParser()
     sub = p.add_subparsers(dest="cmd", required=True)
@@ -103,6 +137,10 @@ def main(argv=None):
     gr = sub.add_parser("grads")
     gr.add_argument("--workload", default=workloads.MLP4096.key, choices=list(workloads.ALL))
     gr.add_argument("--reps", type=int, default=3)
+    rc = sub.add_parser("received")
+    rc.add_argument("--workload", default=workloads.MLP4096.key, choices=list(workloads.ALL))
+    rc.add_argument("--b", type=int, default=64)
+    rc.add_argument("--reps", type=int, default=3)
     args = p.parse_args(argv)
     torch.cuda.set_device(0)
     if args.cmd == "aggregate":
@@ -115,6 +153,8 @@ def main(argv=None):
                 for b in sorted({0, n // 4}):
                     print(json.dumps(aggregate_case(n, d, b, args.reps)), flush=True)
                     torch.cuda.empty_cache()
+    elif args.cmd == "received":
+        print(json.dumps(received_case(args.workload, args.b, args.reps)), flush=True)
     else:
         print(json.dumps(grads_case(args.workload, args.reps)), flush=True)
 

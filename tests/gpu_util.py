@@ -66,42 +66,37 @@ def _rows_close(x, r, rtol, blocks):
         return str(e)
 
 
-def assert_worker_grads_match(G_gpu, loss_gpu, widths, w, X, y, B, bf16, workers, rtol, gpu_active=None,
-                              amb=None):
-    """Each sampled worker's GPU gradient row matches the oracle's Eq. (2) row.
+def oracle_rows_with_decisions(widths, w, X, y, B, bf16, workers, gpu_active=None, amb=None, rows_of=None):
+    """The oracle's Eq. (2) row, loss and magnitude row of each worker in ``workers``,
+    evaluated with the GPU's ReLU decisions where they differ from the oracle's.
 
     A ReLU derivative whose pre-activation lies within rounding of 0 is a
     decision either value of which is correct at the kernel's precision (R13).
     ``gpu_active[h]`` is the GPU's decision set for hidden layer h (its
-    activations > 0, [n*B, width]).  What is unique is checked exactly: every
-    decision the GPU took differently from the oracle must be one the oracle
-    itself certifies as ambiguous (|Z| <= amb * sum of |terms| of that dot
-    product, from the oracle's own pre-activations).  What is then determined is
-    checked with the tolerance: the GPU row against the oracle's Eq. (2) row
-    evaluated with those decisions, relative to the larger of two error scales,
-    the magnitude of the products forming each entry (sum of |terms|: a cancelled
-    sum is only as accurate as its largest terms) and |r| + the rms of the entry's
-    parameter tensor (an entry made of few products inherits the relative error
-    of upstream sums that cancelled).  Returns {worker: (oracle row, oracle loss, magnitude row)}.
+    activations > 0), and ``rows_of(i)`` the rows of worker i in it (default
+    i*B .. i*B+B-1).  Every decision the GPU took differently from the oracle must
+    be one the oracle itself certifies as ambiguous (|Z| <= amb * sum of |terms| of
+    that dot product, from the oracle's own pre-activations); the oracle row is
+    then evaluated with those decisions.  Returns {worker: (row, loss, magnitude)}.
     """
     from oracle import dbw_oracle as O
 
     if amb is None:
         amb = 1e-3 if bf16 else 1e-4
-    blocks = param_blocks(widths)
+    if rows_of is None:
+        def rows_of(i):
+            return slice(i * B, (i + 1) * B)
     L = len(widths) - 1
-    matched, flipped = {}, 0
+    out = {}
     for i in workers:
         Xi, yi = X[i * B:(i + 1) * B], y[i * B:(i + 1) * B]
         g, l, zs, scales, gm = O.worker_grads(widths, w, Xi, yi, 1, B, bf16, return_preact=True,
                                               return_magnitude=True)
-        assert_close_scalar(loss_gpu[i], l[0], rtol, f"loss of worker {i}")
-        flips = None
         if L > 1:
             assert gpu_active is not None and len(gpu_active) == L - 1
             flips = []
             for h in range(L - 1):
-                mine = np.asarray(gpu_active[h][i * B:(i + 1) * B], dtype=bool)
+                mine = np.asarray(gpu_active[h][rows_of(i)], dtype=bool)
                 diff = mine != (zs[h] > 0.0)
                 if diff.any():
                     rel = np.abs(zs[h][diff]) / np.where(scales[h][diff] > 0, scales[h][diff], 1.0)
@@ -109,26 +104,50 @@ def assert_worker_grads_match(G_gpu, loss_gpu, widths, w, X, y, B, bf16, workers
                                                 f"differ from the oracle's outside rounding of 0 "
                                                 f"(largest |Z|/scale {rel.max():.3g})")
                 flips.append(diff)
-                flipped += int(diff.sum())
             if any(f.any() for f in flips):
                 g, _, gm = O.worker_grads(widths, w, Xi, yi, 1, B, bf16, relu_flip=flips, return_magnitude=True)
+        out[i] = (g[0], float(l[0]), gm[0])
+    return out
+
+
+def assert_bf16_close(x, ref, scale, blocks, rtol, what):
+    """bf16-operand result against the oracle: normwise within rtol per parameter
+    tensor (the 2e-2 relative target), and elementwise within rtol of ``scale`` but
+    for a bounded number of bounded outliers: two bf16 rounding chains (fp32 vs fp64
+    values rounded at the same points) drift one bf16 step apart in a growing
+    fraction of deep activations, so a few near-zero entries carry a large relative
+    error."""
+    x = np.asarray(x, dtype=np.float64)
+    r = np.asarray(ref, dtype=np.float64)
+    for (a, b) in blocks:
+        num, den = np.linalg.norm(x[a:b] - r[a:b]), np.linalg.norm(r[a:b])
+        assert num <= rtol * den, f"{what} tensor [{a},{b}): normwise relative error {num / den:.3g}"
+    ratio = np.abs(x - r) / (rtol * scale)
+    nbad = int((ratio > 1.0).sum())
+    assert nbad <= max(1, int(BF16_OUTLIER_FRACTION * x.size)) and ratio.max() <= BF16_OUTLIER_FACTOR, (
+        f"{what}: {nbad} of {x.size} entries beyond 2e-2 of their scale, worst {ratio.max():.3g}x")
+
+
+def assert_worker_grads_match(G_gpu, loss_gpu, widths, w, X, y, B, bf16, workers, rtol, gpu_active=None,
+                              amb=None):
+    """Each sampled worker's GPU gradient row matches the oracle's Eq. (2) row
+    (evaluated with the GPU's certified-ambiguous ReLU decisions, see
+    oracle_rows_with_decisions), relative to the larger of two error scales: the
+    magnitude of the products forming each entry (sum of |terms|: a cancelled sum
+    is only as accurate as its largest terms) and |r| + the rms of the entry's
+    parameter tensor (an entry made of few products inherits the relative error of
+    upstream sums that cancelled).  Returns {worker: (oracle row, oracle loss, magnitude row)}."""
+    blocks = param_blocks(widths)
+    matched = oracle_rows_with_decisions(widths, w, X, y, B, bf16, workers, gpu_active, amb)
+    for i in workers:
+        g, l, gm = matched[i]
+        assert_close_scalar(loss_gpu[i], l, rtol, f"loss of worker {i}")
         x = np.asarray(G_gpu[i], dtype=np.float64)
-        scale = np.maximum(gm[0], tensor_scale(g[0], blocks))
+        scale = np.maximum(gm, tensor_scale(g, blocks))
         if not bf16:
-            assert_close_to_magnitude(x, g[0], scale, rtol, f"G row of worker {i}")
+            assert_close_to_magnitude(x, g, scale, rtol, f"G row of worker {i}")
         else:
-            # normwise per parameter tensor: the 2e-2 relative target
-            for (a, b) in blocks:
-                num, den = np.linalg.norm(x[a:b] - g[0][a:b]), np.linalg.norm(g[0][a:b])
-                assert num <= rtol * den, f"worker {i} tensor [{a},{b}): normwise relative error {num / den:.3g}"
-            # elementwise bug detector: two bf16 rounding chains (fp32 vs fp64 values rounded
-            # at the same points) drift one bf16 step apart in a growing fraction of deep
-            # activations, so a few near-zero activations carry a large relative error
-            ratio = np.abs(x - g[0]) / (rtol * scale)
-            nbad = int((ratio > 1.0).sum())
-            assert nbad <= max(1, int(BF16_OUTLIER_FRACTION * x.size)) and ratio.max() <= BF16_OUTLIER_FACTOR, (
-                f"worker {i}: {nbad} of {x.size} entries beyond 2e-2 of their scale, worst {ratio.max():.3g}x")
-        matched[i] = (g[0], float(l[0]), gm[0])
+            assert_bf16_close(x, g, scale, blocks, rtol, f"worker {i}")
     return matched
 
 

@@ -79,3 +79,28 @@ def test_host_validation_rejects_before_launch(lib):
     L, arr = dbw._widths([784, 10])
     assert lib.dbw_worker_grads(L, arr, 0, 256, 7850, 256, 10, 256, 256, 16, 32, 256, 7850, 256, 256, 1 << 20,
                                 null) == dbw.DBW_EALIGN   # ld % 4 != 0
+
+
+def test_received_form_queries(lib):
+    """The received-workers form: workspace only for the shapes it supports (bf16,
+    B % 32 == 0, B | 128 or 128 | B), at least the per-worker pass's workspace (it
+    extends that layout); a partials buffer of one block per quantity; host checks."""
+    widths = [4096, 4096, 4096, 4096, 1000]
+    full = dbw.dbw_worker_grads_workspace_bytes(widths, 256, 32, dbw.PREC_BF16)
+    rx = dbw.dbw_received_grads_workspace_bytes(widths, 256, 32, dbw.PREC_BF16)
+    assert rx > full > 0
+    for n, B in ((128, 128), (4, 256), (8, 64)):
+        assert dbw.dbw_received_grads_workspace_bytes([3072, 1024, 1024, 10], n, B, dbw.PREC_BF16) > 0
+    assert dbw.dbw_received_grads_workspace_bytes(widths, 256, 32, dbw.PREC_FP32) == 0
+    assert dbw.dbw_received_grads_workspace_bytes(widths, 256, 96, dbw.PREC_BF16) == 0
+    assert dbw.dbw_received_grads_workspace_bytes(widths, 256, 16, dbw.PREC_BF16) == 0
+    assert dbw.dbw_received_partials_bytes(16) == 8 * (4 + 2 * 18)
+    assert dbw.dbw_received_partials_bytes(0) == 0 and dbw.dbw_received_partials_bytes(dbw.NMAX + 1) == 0
+    L, arr = dbw._widths([784, 10])
+    null = None
+    args = [L, arr, dbw.PREC_BF16, 256, 7850, 256, 10, 256, 256, 16, 32, 256, C.c_float(0.1), null, 256, 256]
+    assert lib.dbw_received_grads_update(*args, 1 << 20, 256, 1 << 30, null) != dbw.DBW_OK   # no device here
+    assert lib.dbw_received_grads_update(*args[:3], null, *args[4:], 1 << 20, 256, 1 << 30, null) == dbw.DBW_EINVAL
+    assert lib.dbw_received_grads_update(*args, 16, 256, 1 << 30, null) == dbw.DBW_EINVAL          # partials too small
+    args[3] = 260
+    assert lib.dbw_received_grads_update(*args, 1 << 20, 256, 1 << 30, null) == dbw.DBW_EALIGN
