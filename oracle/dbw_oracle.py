@@ -420,17 +420,21 @@ def _ieee_div(a, b):
         return float(np.float64(a) / np.float64(b))
 
 
-def choose_k(st: State, lr, beta, blind=False):
+def choose_k(st: State, lr, beta, blind=False, T=None):
     """Eqs. (18)-(19): k_t for the iteration about to start; returns (k_t, ratio list).
 
     ``blind`` is the paper's B-DBW variant (Sect. 4): the gain is k itself.
+    ``T`` replaces the push-and-interrupt time estimates S_k / c by given T^_k
+    (the push-and-wait estimator of Eq. (17)); NaN estimates mean "none yet".
     """
     n = st.n
     ratio = [math.nan] * n
     kstar = n
+    have_T = (st.c > 0) if T is None else (not math.isnan(T[0]))
+    if T is None and st.c > 0:
+        T = time_estimates(st)
     if blind:
-        if st.c > 0:
-            T = time_estimates(st)
+        if have_T:
             best = -math.inf
             for k in range(1, n + 1):
                 ratio[k - 1] = _ieee_div(float(k), T[k - 1])
@@ -438,8 +442,7 @@ def choose_k(st: State, lr, beta, blind=False):
                     best, kstar = ratio[k - 1], k
     else:
         gains = gain_estimates(st, lr)
-        if gains is not None:
-            T = time_estimates(st)
+        if gains is not None and have_T:
             best = -math.inf
             found = False
             for k in range(1, n + 1):
