@@ -13,6 +13,9 @@
  *   dbw_grad_stats        Eqs. (10)-(12) and Sect. 3.2: finishes the statistics
  *                         and records them (and the order statistics) in the state
  *
+ * Push-and-wait clock and the time estimator of Eq. (17) (Sect. 2, 3.2):
+ *   dbw_psw_arrivals / dbw_psw_record / dbw_psw_estimate, dbw_choose_b_times
+ *
  * A second form of the iteration skips the [n, d] matrix:
  *   dbw_received_grads_update  Eqs. (2)-(4) and the partial sums of Eqs. (10)-(11)
  *                         for the received workers only (replaces dbw_worker_grads +
@@ -372,6 +375,97 @@ int dbw_grad_stats(const double* partials, int n, const uint8_t* mask,
  */
 int dbw_choose_b(dbw_state* state, double lr, double beta, int flags,
                  int32_t* b_out, double* ratio_out, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Push-and-wait (PsW, Sect. 2): after an update the PS pushes the new vector; a
+ * busy worker first completes its current computation, then takes the most
+ * recent vector.  The k_{t-1} workers received last time are idle when
+ * iteration t starts, the others are still busy for a residual time r_j.
+ * Sect. 3.2: t_{h,i,t} = time, from the start of iteration t, at which the i-th
+ * gradient of w_t arrives given k_{t-1} = h; late workers still report, so
+ * every worker that computes on w_t yields a sample (when it arrives).
+ * Eq. (17): x_{h,k} = least squares fit to the samples of cell (h, k), increasing
+ * in k, decreasing in h, increasing along the diagonal; T^_k = x*_{k,k}.
+ *
+ * Readings (the paper leaves these open):
+ *  - worker j's round trip time on w_t is omega_j of iteration t (one
+ *    computation per worker per iteration); it computes on w_t iff r_j < T_t,
+ *    where T_t is the k_t-th arrival; its gradient then arrives at r_j + omega_j.
+ *  - Eq. (17) does not fix cells without samples.  The rows whose diagonal cell
+ *    has samples are fitted on their observed cells, weighted by sample counts.
+ *    A row's observed ranks are a prefix, so chains over observed cells generate
+ *    the order among them.  Every other diagonal cell is the pooled mean of its
+ *    column, made nondecreasing over such cells and clipped to the bounds the
+ *    order places on it.  No such row yet: T^ is NaN.
+ *  - the fit is Dykstra's alternating projections with weighted
+ *    pool-adjacent-violators on each chain, in fp32 (sample counts and sums are
+ *    exact; fp64 would cost ~14x in the sequential chains), warm-started from the
+ *    previous estimate's dual variables, stopped when a sweep moves no cell by
+ *    more than tol x the largest cell mean.
+ *
+ * The state is one opaque device buffer of dbw_psw_bytes(n) bytes that starts
+ * with this header (the offsets locate its arrays, for inspection):
+ */
+typedef struct {
+    int32_t n;          /* workers */
+    int32_t h;          /* k_{t-1} (n before the first iteration) */
+    int32_t sweeps;     /* Dykstra sweeps of the last dbw_psw_estimate */
+    int32_t flags;      /* DBW_PSW_* bits, sticky */
+    double vclock;      /* tau_t, the push-and-wait virtual clock */
+    double unit;        /* value of one unit of the int64 cell sums (2^-32) */
+    int64_t iterations; /* iterations recorded */
+    int64_t off_r;      /* double  r[n]        residual busy time of each worker */
+    int64_t off_pend;   /* int32   pend[2n]    (h, i) of worker j's sample still on its way, h = 0: none */
+    int64_t off_pendv;  /* double  pendv[n]    its value */
+    int64_t off_sum;    /* int64   sum[n*n]    cell (h, i) at (h-1)*n + (i-1), in units */
+    int64_t off_cnt;    /* int32   cnt[n*n]    samples of each cell */
+    int64_t off_x;      /* float   x[n*n]      fitted cells of the group rows (fp32 fit) */
+    int64_t reserved[6];
+} dbw_psw_header;
+
+#define DBW_PSW_NOT_CONVERGED 1 /* the last estimate stopped at max_sweeps */
+#define DBW_PSW_RANGE 2         /* a sample outside [0, 2^31) was clamped in the cell sums */
+
+/* Bytes of the push-and-wait state for n workers (grows as n^2: 5.3 MB at n = 256, 84 MB at n = 1024). */
+size_t dbw_psw_bytes(int n);
+
+/* All workers idle, no sample, tau = 0, h = n.  psw: 256-byte aligned device buffer. */
+int dbw_psw_init(void* psw, int n, void* stream);
+
+/*
+ * arrivals[j] = r_j + omega[j]: when worker j's gradient of w_t reaches the PS,
+ * counted from the start of iteration t.  Pass ``arrivals`` to
+ * dbw_select_fastest as the times: its first k_t are the received workers.
+ *  omega  [n] fp64 this iteration's round trip times (device).
+ */
+int dbw_psw_arrivals(const void* psw, int n, const double* omega, double* arrivals, void* stream);
+
+/*
+ * End of iteration t: with T_t = tsorted[k-1], records every sample that has
+ * reached the PS (the arrivals up to T_t, and earlier late samples whose worker
+ * became free), keeps the later ones pending, advances the residuals, the clock
+ * (tau += T_t) and h = k_t.
+ *  order, tsorted, k   from the dbw_select_fastest call on dbw_psw_arrivals' output.
+ */
+int dbw_psw_record(void* psw, int n, const int32_t* order, const double* tsorted, const int32_t* k,
+                   void* stream);
+
+/*
+ * Eq. (17): T_hat[k-1] = T^_k for k = 1..n (NaN before any sample).
+ *  tol         stop when a Dykstra sweep moves no cell by more than tol x the
+ *              largest cell mean; > 0, values below 1e-6 (the fp32 fit's
+ *              resolution) act as 1e-6.
+ *  max_sweeps  cap (>= 1); reaching it raises DBW_PSW_NOT_CONVERGED.
+ */
+int dbw_psw_estimate(void* psw, int n, double tol, int max_sweeps, double* T_hat, void* stream);
+
+/*
+ * dbw_choose_b with given time estimates: T^_k = T_hat[k-1] in Eqs. (18)-(19)
+ * instead of the push-and-interrupt S[k-1] / c (e.g. dbw_psw_estimate's output).
+ * NaN in T_hat[0] means "no estimate yet": k_t = n.
+ */
+int dbw_choose_b_times(dbw_state* state, const double* T_hat, double lr, double beta, int flags, int32_t* b_out,
+                       double* ratio_out, void* stream);
 
 #ifdef __cplusplus
 }

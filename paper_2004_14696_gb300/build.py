@@ -23,7 +23,7 @@ LIB = os.path.join(PKG, "libdbw.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC,
           "--expt-relaxed-constexpr"]
-PER_FILE = {"estimator.cu": ["-fmad=false"]}
+PER_FILE = {"estimator.cu": ["-fmad=false"], "psw.cu": ["-fmad=false"]}
 
 
 def nvcc() -> str:

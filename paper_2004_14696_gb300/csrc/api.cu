@@ -217,8 +217,76 @@ int dbw_choose_b(dbw_state* state, double lr, double beta, int flags, int32_t* b
     if (!aligned16(state)) return fail(DBW_EALIGN, "dbw_choose_b: state must be 16-byte aligned");
     int rc = check_device();
     if (rc) return rc;
-    cudaError_t e = launch_choose_b(state, lr, beta, flags, b_out, ratio_out, as_stream(stream));
+    cudaError_t e = launch_choose_b(state, lr, beta, flags, b_out, ratio_out, nullptr, as_stream(stream));
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_choose_b: %s", cudaGetErrorString(e));
+    return DBW_OK;
+}
+
+int dbw_choose_b_times(dbw_state* state, const double* T_hat, double lr, double beta, int flags, int32_t* b_out,
+                       double* ratio_out, void* stream) {
+    g_err[0] = 0;
+    if (!state || !T_hat || !b_out) return fail(DBW_EINVAL, "dbw_choose_b_times: NULL pointer argument");
+    if (!(lr > 0.0)) return fail(DBW_EINVAL, "dbw_choose_b_times: lr must be > 0");
+    if (!(beta >= 1.0)) return fail(DBW_EINVAL, "dbw_choose_b_times: beta must be >= 1");
+    if (flags & ~DBW_CHOOSE_BLIND) return fail(DBW_EINVAL, "dbw_choose_b_times: unknown flags");
+    if (!aligned16(state)) return fail(DBW_EALIGN, "dbw_choose_b_times: state must be 16-byte aligned");
+    int rc = check_device();
+    if (rc) return rc;
+    cudaError_t e = launch_choose_b(state, lr, beta, flags, b_out, ratio_out, T_hat, as_stream(stream));
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_choose_b_times: %s", cudaGetErrorString(e));
+    return DBW_OK;
+}
+
+size_t dbw_psw_bytes(int n) {
+    if (n < 1 || n > DBW_NMAX) return 0;
+    return psw_bytes(n);
+}
+
+static int psw_args(const char* what, const void* psw, int n) {
+    if (!psw) return fail(DBW_EINVAL, "%s: NULL state", what);
+    if (n < 1 || n > DBW_NMAX) return fail(DBW_EINVAL, "%s: n must be in [1, %d]", what, DBW_NMAX);
+    if (!aligned256(psw)) return fail(DBW_EALIGN, "%s: state must be 256-byte aligned", what);
+    return check_device();
+}
+
+int dbw_psw_init(void* psw, int n, void* stream) {
+    g_err[0] = 0;
+    int rc = psw_args("dbw_psw_init", psw, n);
+    if (rc) return rc;
+    cudaError_t e = launch_psw_init(psw, n, as_stream(stream));
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_psw_init: %s", cudaGetErrorString(e));
+    return DBW_OK;
+}
+
+int dbw_psw_arrivals(const void* psw, int n, const double* omega, double* arrivals, void* stream) {
+    g_err[0] = 0;
+    if (!omega || !arrivals) return fail(DBW_EINVAL, "dbw_psw_arrivals: NULL pointer argument");
+    int rc = psw_args("dbw_psw_arrivals", psw, n);
+    if (rc) return rc;
+    cudaError_t e = launch_psw_arrivals(psw, n, omega, arrivals, as_stream(stream));
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_psw_arrivals: %s", cudaGetErrorString(e));
+    return DBW_OK;
+}
+
+int dbw_psw_record(void* psw, int n, const int32_t* order, const double* tsorted, const int32_t* k, void* stream) {
+    g_err[0] = 0;
+    if (!order || !tsorted || !k) return fail(DBW_EINVAL, "dbw_psw_record: NULL pointer argument");
+    int rc = psw_args("dbw_psw_record", psw, n);
+    if (rc) return rc;
+    cudaError_t e = launch_psw_record(psw, n, order, tsorted, k, as_stream(stream));
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_psw_record: %s", cudaGetErrorString(e));
+    return DBW_OK;
+}
+
+int dbw_psw_estimate(void* psw, int n, double tol, int max_sweeps, double* T_hat, void* stream) {
+    g_err[0] = 0;
+    if (!T_hat) return fail(DBW_EINVAL, "dbw_psw_estimate: NULL T_hat");
+    if (!(tol > 0.0)) return fail(DBW_EINVAL, "dbw_psw_estimate: tol must be > 0");
+    if (max_sweeps < 1) return fail(DBW_EINVAL, "dbw_psw_estimate: max_sweeps must be >= 1");
+    int rc = psw_args("dbw_psw_estimate", psw, n);
+    if (rc) return rc;
+    cudaError_t e = launch_psw_estimate(psw, n, tol, max_sweeps, T_hat, as_stream(stream));
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_psw_estimate: %s", cudaGetErrorString(e));
     return DBW_OK;
 }
 

@@ -44,7 +44,15 @@ cudaError_t launch_grad_stats(const double* partials, int n, const uint8_t* mask
                               const double* tsorted, double lr, dbw_state* s, double* stats_out,
                               double* row_sqnorm, cudaStream_t st);
 cudaError_t launch_choose_b(dbw_state* s, double lr, double beta, int flags, int32_t* b_out,
-                            double* ratio_out, cudaStream_t st);
+                            double* ratio_out, const double* T_ext, cudaStream_t st);
+
+// Push-and-wait clock and Eq. (17) (psw.cu)
+size_t psw_bytes(int n);
+cudaError_t launch_psw_init(void* psw, int n, cudaStream_t st);
+cudaError_t launch_psw_arrivals(const void* psw, int n, const double* omega, double* e, cudaStream_t st);
+cudaError_t launch_psw_record(void* psw, int n, const int32_t* order, const double* tsorted, const int32_t* k,
+                              cudaStream_t st);
+cudaError_t launch_psw_estimate(void* psw, int n, double tol, int max_sweeps, double* T_hat, cudaStream_t st);
 
 // Worker gradients (grads.cu)
 struct GradsPlan;

@@ -135,9 +135,12 @@ __global__ void __launch_bounds__(1024) grad_stats_kernel(
         for (int j = tid; j < n; j += blockDim.x) row_sqnorm[j] = mask[j] ? sums[j] : CUDART_NAN;
 }
 
+// T_ext (nullable): time estimates T^_k = T_ext[k-1] instead of S[k-1] / c; NaN in
+// T_ext[0] means no estimate yet.
 __global__ void __launch_bounds__(1024) choose_b_kernel(dbw_state* __restrict__ st, double lr, double beta,
                                                         int flags, int32_t* __restrict__ b_out,
-                                                        double* __restrict__ ratio_out) {
+                                                        double* __restrict__ ratio_out,
+                                                        const double* __restrict__ T_ext) {
     __shared__ double Vh_s, Nh_s, q_s;
     __shared__ int ready_s;
     __shared__ double best_r[32];
@@ -152,10 +155,11 @@ __global__ void __launch_bounds__(1024) choose_b_kernel(dbw_state* __restrict__ 
     const bool blind = (flags & DBW_CHOOSE_BLIND) != 0;
     if (tid == 0) {
         int ready;
+        const bool have_T = T_ext ? !isnan(T_ext[0]) : st->c > 0;
         if (blind) {
-            ready = st->c > 0;
+            ready = have_T;
         } else {
-            ready = st->cntV > 0 && st->cntN > 0 && st->cntL > 0 && st->c > 0;
+            ready = st->cntV > 0 && st->cntN > 0 && st->cntL > 0 && st->c > 0 && have_T;
             if (ready) {
                 Vh_s = window_mean(st->ringV, st->cntV, st->D);   // Eq. (13)
                 Nh_s = window_mean(st->ringN, st->cntN, st->D);   // Eq. (14)
@@ -175,7 +179,7 @@ __global__ void __launch_bounds__(1024) choose_b_kernel(dbw_state* __restrict__ 
         double ratio = CUDART_NAN;
         bool elig = false;
         if (ready) {
-            const double T = st->S[k - 1] / c;                    // T^_k
+            const double T = T_ext ? T_ext[k - 1] : st->S[k - 1] / c;   // T^_k
             if (blind) {
                 ratio = (double)k / T;
                 elig = true;
@@ -262,8 +266,8 @@ cudaError_t launch_grad_stats(const double* partials, int n, const uint8_t* mask
 }
 
 cudaError_t launch_choose_b(dbw_state* s, double lr, double beta, int flags, int32_t* b_out,
-                            double* ratio_out, cudaStream_t st) {
-    choose_b_kernel<<<1, 1024, 0, st>>>(s, lr, beta, flags, b_out, ratio_out);
+                            double* ratio_out, const double* T_ext, cudaStream_t st) {
+    choose_b_kernel<<<1, 1024, 0, st>>>(s, lr, beta, flags, b_out, ratio_out, T_ext);
     return cudaGetLastError();
 }
 

@@ -11,6 +11,7 @@ from __future__ import annotations
 import ctypes as C
 import os
 
+import numpy as np
 import torch
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
@@ -21,9 +22,20 @@ PREC_FP32, PREC_BF16 = 0, 1
 NMAX, DMAX, LMAX = 1024, 64, 8
 CHOOSE_BLIND = 1
 FLAG_K1, FLAG_L_SKIPPED, FLAG_EMPTY_MASK, FLAG_BAD_STATE = 1, 2, 4, 8
+PSW_NOT_CONVERGED, PSW_RANGE = 1, 2
 STAT_K, STAT_SS, STAT_GBAR_SQ, STAT_V, STAT_N, STAT_F, STAT_L, STAT_FLAGS, STAT_VCLOCK = range(9)
 STATS_LEN = 9
 PARTIALS_MAGIC = 0x44425750415254
+
+
+class PswHeader(C.Structure):
+    """Mirror of ``dbw_psw_header`` (the start of the push-and-wait state buffer)."""
+    _fields_ = [
+        ("n", C.c_int32), ("h", C.c_int32), ("sweeps", C.c_int32), ("flags", C.c_int32),
+        ("vclock", C.c_double), ("unit", C.c_double), ("iterations", C.c_int64),
+        ("off_r", C.c_int64), ("off_pend", C.c_int64), ("off_pendv", C.c_int64), ("off_sum", C.c_int64),
+        ("off_cnt", C.c_int64), ("off_x", C.c_int64), ("reserved", C.c_int64 * 6),
+    ]
 
 
 class DbwState(C.Structure):
@@ -67,6 +79,12 @@ _SIGS = {
     "dbw_received_partials_bytes": (_sz, [_i32]),
     "dbw_received_grads_update": (_i32, [_i32, _vp, _i32, _vp, _i64, _vp, _i64, _vp, _vp, _i32, _i32, _vp, _f32,
                                          _vp, _vp, _vp, _sz, _vp, _sz, _vp]),
+    "dbw_psw_bytes": (_sz, [_i32]),
+    "dbw_psw_init": (_i32, [_vp, _i32, _vp]),
+    "dbw_psw_arrivals": (_i32, [_vp, _i32, _vp, _vp, _vp]),
+    "dbw_psw_record": (_i32, [_vp, _i32, _vp, _vp, _vp, _vp]),
+    "dbw_psw_estimate": (_i32, [_vp, _i32, _f64, _i32, _vp, _vp]),
+    "dbw_choose_b_times": (_i32, [_vp, _vp, _f64, _f64, _i32, _vp, _vp, _vp]),
     "dbw_state_init": (_i32, [_vp, _i32, _i32, _vp]),
     "dbw_grad_stats": (_i32, [_vp, _i32, _vp, _vp, _vp, _f64, _vp, _vp, _vp, _vp]),
     "dbw_choose_b": (_i32, [_vp, _f64, _f64, _i32, _vp, _vp, _vp]),
@@ -188,6 +206,63 @@ def dbw_received_grads_update(widths, prec, w, pool, labels, idx, n, B, mask, lr
         _ptr(partials, torch.uint8, "partials"), partials.numel(), _ptr(ws, torch.uint8, "ws"), ws.numel(),
         _stream(stream))
     _check("dbw_received_grads_update", rc)
+
+
+def dbw_psw_bytes(n):
+    return int(lib().dbw_psw_bytes(n))
+
+
+def dbw_psw_init(psw, n, stream=None):
+    _check("dbw_psw_init", lib().dbw_psw_init(_ptr(psw, torch.uint8, "psw"), n, _stream(stream)))
+
+
+def dbw_psw_arrivals(psw, n, omega, arrivals, stream=None):
+    rc = lib().dbw_psw_arrivals(_ptr(psw, torch.uint8, "psw"), n, _ptr(omega, torch.float64, "omega"),
+                                _ptr(arrivals, torch.float64, "arrivals"), _stream(stream))
+    _check("dbw_psw_arrivals", rc)
+
+
+def dbw_psw_record(psw, n, order, tsorted, k, stream=None):
+    rc = lib().dbw_psw_record(_ptr(psw, torch.uint8, "psw"), n, _ptr(order, torch.int32, "order"),
+                              _ptr(tsorted, torch.float64, "tsorted"), _ptr(k, torch.int32, "k"), _stream(stream))
+    _check("dbw_psw_record", rc)
+
+
+def dbw_psw_estimate(psw, n, T_hat, tol=1e-6, max_sweeps=100000, stream=None):
+    rc = lib().dbw_psw_estimate(_ptr(psw, torch.uint8, "psw"), n, float(tol), int(max_sweeps),
+                                _ptr(T_hat, torch.float64, "T_hat"), _stream(stream))
+    _check("dbw_psw_estimate", rc)
+
+
+def dbw_choose_b_times(state, T_hat, lr, beta, b_out, ratio_out=None, flags=0, stream=None):
+    rc = lib().dbw_choose_b_times(_ptr(state, torch.uint8, "state"), _ptr(T_hat, torch.float64, "T_hat"), float(lr),
+                                  float(beta), int(flags), _ptr(b_out, torch.int32, "b_out"),
+                                  _ptr(ratio_out, torch.float64, "ratio_out", nullable=True), _stream(stream))
+    _check("dbw_choose_b_times", rc)
+
+
+def new_psw(n, device="cuda", stream=None):
+    """A device push-and-wait state buffer for n workers, initialised."""
+    t = torch.empty(dbw_psw_bytes(n), dtype=torch.uint8, device=device)
+    dbw_psw_init(t, n, stream)
+    return t
+
+
+def read_psw(psw, n):
+    """Host copy of the push-and-wait state: header fields and its arrays (synchronises)."""
+    raw = psw.cpu().numpy()
+    hdr = PswHeader.from_buffer_copy(raw[:C.sizeof(PswHeader)].tobytes())
+    nn = n * n
+
+    def arr(off, dtype, count):
+        return np.frombuffer(raw[off:off + count * np.dtype(dtype).itemsize].tobytes(), dtype=dtype)
+    pend = arr(hdr.off_pend, np.int32, 2 * n).reshape(n, 2)
+    return {"n": hdr.n, "h": hdr.h, "sweeps": hdr.sweeps, "flags": hdr.flags, "vclock": hdr.vclock,
+            "iterations": hdr.iterations, "r": arr(hdr.off_r, np.float64, n),
+            "pend": pend, "pendv": arr(hdr.off_pendv, np.float64, n),
+            "sums": arr(hdr.off_sum, np.uint64, nn).reshape(n, n).astype(np.float64) * hdr.unit,
+            "sums_raw": arr(hdr.off_sum, np.uint64, nn).reshape(n, n),
+            "cnts": arr(hdr.off_cnt, np.int32, nn).reshape(n, n), "x": arr(hdr.off_x, np.float32, nn).reshape(n, n)}
 
 
 def dbw_select_fastest(times, b, order, mask, tsorted, k_out=None, stream=None):

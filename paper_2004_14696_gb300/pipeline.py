@@ -26,7 +26,8 @@ from .workloads import Workload
 
 class Iteration:
     def __init__(self, wl: Workload, device="cuda", static_b=None, blind=False, keep_gbar=False,
-                 pool=None, labels=None, w0=None, received=False):
+                 pool=None, labels=None, w0=None, received=False, clock="psi", psw_tol=1e-6,
+                 psw_max_sweeps=100000):
         self.wl = wl
         self.device = torch.device(device)
         n, d, ld = wl.n, wl.d, wl.ld
@@ -34,6 +35,10 @@ class Iteration:
         self.static_b = static_b
         self.blind = blind
         self.received = received
+        if clock not in ("psi", "psw"):
+            raise ValueError("clock must be 'psi' (push-and-interrupt) or 'psw' (push-and-wait)")
+        self.clock = clock
+        self.psw_tol, self.psw_max_sweeps = psw_tol, psw_max_sweeps
         if pool is None:
             pool = inputs.feature_pool(wl.seed, wl.S, wl.widths[0], wl.feature_dist)
         if labels is None:
@@ -69,6 +74,10 @@ class Iteration:
         self.stats = torch.empty(dbw.STATS_LEN, dtype=torch.float64, device=self.device)
         self.row_sqnorm = torch.empty(n, dtype=torch.float64, device=self.device)
         self.gbar = torch.empty(d, dtype=torch.float32, device=self.device) if keep_gbar else None
+        if clock == "psw":
+            self.psw = dbw.new_psw(n, self.device)
+            self.T_hat = torch.full((n,), float("nan"), dtype=torch.float64, device=self.device)
+            self.arrivals = torch.empty(n, dtype=torch.float64, device=self.device)
         # per-step inputs (device copies written by the caller or by load_inputs)
         self.idx = torch.empty(n * wl.B, dtype=torch.int32, device=self.device)
         self.times = torch.empty(n, dtype=torch.float64, device=self.device)
@@ -91,11 +100,20 @@ class Iteration:
         wl = self.wl
         idx = self.idx if idx is None else idx
         times = self.times if times is None else times
+        psw = self.clock == "psw"
         if self.static_b is None:
-            dbw.dbw_choose_b(self.state, wl.lr, wl.beta, self.b, self.ratio,
-                             dbw.CHOOSE_BLIND if self.blind else 0, stream)
+            if psw:
+                dbw.dbw_choose_b_times(self.state, self.T_hat, wl.lr, wl.beta, self.b, self.ratio,
+                                       dbw.CHOOSE_BLIND if self.blind else 0, stream)
+            else:
+                dbw.dbw_choose_b(self.state, wl.lr, wl.beta, self.b, self.ratio,
+                                 dbw.CHOOSE_BLIND if self.blind else 0, stream)
         # static b is known on the host: its learning-rate rule applies; DBW uses lr
         lr = wl.lr if self.static_b is None else wl.lr_for(wl.n - int(self.static_b))
+        if psw:
+            # push-and-wait: the gradients of w_t arrive at the residual busy time plus the round trip
+            dbw.dbw_psw_arrivals(self.psw, wl.n, times, self.arrivals, stream)
+            times = self.arrivals
         if self.received:
             dbw.dbw_select_fastest(times, self.b, self.order, self.mask, self.tsorted, self.k, stream)
             dbw.dbw_received_grads_update(wl.widths, wl.prec, self.w, self.pool, self.labels, idx, wl.n, wl.B,
@@ -107,6 +125,9 @@ class Iteration:
             dbw.dbw_aggregate_update(self.G, wl.n, self.d, self.mask, lr, self.w, self.partials, self.gbar, stream)
         dbw.dbw_grad_stats(self.partials, wl.n, self.mask, self.loss, self.tsorted, lr, self.state, self.stats,
                            self.row_sqnorm, stream)
+        if psw:
+            dbw.dbw_psw_record(self.psw, wl.n, self.order, self.tsorted, self.k, stream)
+            dbw.dbw_psw_estimate(self.psw, wl.n, self.T_hat, self.psw_tol, self.psw_max_sweeps, stream)
 
     # ------------------------------------------------------------ checkpoint
     def checkpoint(self):
@@ -116,8 +137,12 @@ class Iteration:
         iteration rewrites, so (w, state) restores the run exactly.
         """
         torch.cuda.synchronize(self.device)
-        return {"w": self.w.detach().cpu().clone(), "state": self.state.detach().cpu().clone(),
-                "b": self.b.detach().cpu().clone(), "key": self.wl.key}
+        ck = {"w": self.w.detach().cpu().clone(), "state": self.state.detach().cpu().clone(),
+              "b": self.b.detach().cpu().clone(), "key": self.wl.key}
+        if self.clock == "psw":
+            ck["psw"] = self.psw.detach().cpu().clone()
+            ck["T_hat"] = self.T_hat.detach().cpu().clone()
+        return ck
 
     def restore(self, ckpt):
         if ckpt["key"] != self.wl.key:
@@ -125,6 +150,9 @@ class Iteration:
         self.w.copy_(ckpt["w"])
         self.state.copy_(ckpt["state"])
         self.b.copy_(ckpt["b"])
+        if self.clock == "psw":
+            self.psw.copy_(ckpt["psw"])
+            self.T_hat.copy_(ckpt["T_hat"])
 
     def record(self, t, wall_ms=None):
         """One iteration's log record (reads the statistics back: synchronises)."""
@@ -142,7 +170,7 @@ class Iteration:
     def launches_per_step(self):
         """Kernels libdbw launches per step (for the bench's launch count)."""
         L = len(self.wl.widths) - 1
-        choose = 0 if self.static_b is not None else 1
+        choose = (0 if self.static_b is not None else 1) + (3 if self.clock == "psw" else 0)   # + arrivals, record, fit
         if self.received:
             # select; status memset, compaction, L weight cast-transposes, gather + X^T, L forward
             # GEMMs, loss + dZ^T, per layer (mean-gradient GEMM, bias sums, bias update, Gram),
@@ -169,7 +197,7 @@ def agg_case(n, d, seed, b, device="cuda", mean=0.0, std=1.0):
 
 
 def run(wl: Workload, iters, log=None, static_b=None, blind=False, device="cuda", start=0, it=None,
-        received=False):
+        received=False, clock="psi"):
     """Run ``iters`` iterations of a workload; returns (and optionally writes as JSON
     lines to the file object ``log``) one record per iteration: b_t, k_t, the k_t-th
     arrival time T_(k_t) (the iteration's virtual duration), the virtual clock, F^_t,
@@ -177,7 +205,7 @@ def run(wl: Workload, iters, log=None, static_b=None, blind=False, device="cuda"
     import json
     import time
     if it is None:
-        it = Iteration(wl, device=device, static_b=static_b, blind=blind, received=received)
+        it = Iteration(wl, device=device, static_b=static_b, blind=blind, received=received, clock=clock)
     out = []
     for t in range(start, start + iters):
         it.load_inputs(t)
@@ -202,12 +230,14 @@ def _main(argv=None):
     p.add_argument("--blind", action="store_true", help="B-DBW: the gain of k is k itself")
     p.add_argument("--received", action="store_true",
                    help="received workers only, without the [n, d] gradient matrix")
+    p.add_argument("--clock", default="psi", choices=["psi", "psw"],
+                   help="push-and-interrupt (fresh times) or push-and-wait (residual times, Eq. (17) estimator)")
     p.add_argument("--log", default="-")
     a = p.parse_args(argv)
     wl = workloads.ALL[a.workload]
     f = sys.stdout if a.log == "-" else open(a.log, "w")
     try:
-        run(wl, a.iters or wl.iters, f, a.static_b, a.blind, received=a.received)
+        run(wl, a.iters or wl.iters, f, a.static_b, a.blind, received=a.received, clock=a.clock)
     finally:
         if f is not sys.stdout:
             f.close()

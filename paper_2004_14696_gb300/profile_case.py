@@ -4,6 +4,7 @@
     python -m paper_2004_14696_gb300.profile_case sweep            # the aggregation-only sweep
     python -m paper_2004_14696_gb300.profile_case grads --workload mlp4096x3-1000_n256_B32 --reps 3
     python -m paper_2004_14696_gb300.profile_case received --workload mlp4096x3-1000_n256_B32 --b 64
+    python -m paper_2004_14696_gb300.profile_case psw --n 256 --iters 60     # push-and-wait clock + Eq. (17)
 
 Each prints one JSON line per case with CUDA-event times (on the launching
 stream, after warm-up).  Large gradient matrices are filled on the device with
@@ -123,6 +124,50 @@ def received_case(key, b, reps, warmup=2):
             "status": int(it.ws[:4].view(torch.int32).item())}
 
 
+def psw_case(n, iters, seed=2004146971, model="pareto", tol=1e-6):
+    """The push-and-wait clock and the Eq. (17) fit alone, per iteration: arrivals,
+    selection, record and the warm-started fit, with k_t drawn uniformly from 1..n
+    (every row of the cell table gets samples, the hardest case for the fit)."""
+    psw = dbw.new_psw(n)
+    e = torch.empty(n, dtype=torch.float64, device="cuda")
+    T = torch.empty(n, dtype=torch.float64, device="cuda")
+    bt = torch.zeros(1, dtype=torch.int32, device="cuda")
+    order = torch.empty(n, dtype=torch.int32, device="cuda")
+    mask = torch.empty(n, dtype=torch.uint8, device="cuda")
+    ts = torch.empty(n, dtype=torch.float64, device="cuda")
+    kk = torch.empty(1, dtype=torch.int32, device="cuda")
+    rng = np.random.default_rng(seed)
+    om = torch.from_numpy(np.stack([inputs.completion_times(seed, t, n, model, alpha=2.0, xm=1.0)
+                                    for t in range(iters)])).cuda()
+    bs = torch.from_numpy(np.array([0] + [n - int(rng.integers(1, n + 1)) for _ in range(iters - 1)],
+                                   dtype=np.int32)).cuda()
+    st = torch.cuda.current_stream()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(iters)]
+    sweeps = []
+    for t in range(iters):
+        ev[t][0].record(st)
+        dbw.dbw_psw_arrivals(psw, n, om[t], e)
+        bt.copy_(bs[t:t + 1])
+        dbw.dbw_select_fastest(e, bt, order, mask, ts, kk)
+        dbw.dbw_psw_record(psw, n, order, ts, kk)
+        ev[t][1].record(st)
+        dbw.dbw_psw_estimate(psw, n, T, tol=tol)
+        ev[t][2].record(st)
+        sweeps.append(psw[8:12].clone())   # dbw_psw_header.sweeps (int32 at byte 8)
+    torch.cuda.synchronize()
+    clock_ms = [ev[t][0].elapsed_time(ev[t][1]) for t in range(iters)]
+    fit_ms = [ev[t][1].elapsed_time(ev[t][2]) for t in range(iters)]
+    sw = [int(x.view(torch.int32).item()) for x in sweeps]
+    h = dbw.read_psw(psw, n)
+    rows = int((h["cnts"].sum(axis=1) > 0).sum())
+    tail = slice(iters // 2, iters)
+    return {"case": "psw", "n": n, "iters": iters, "tol": tol, "data_rows_at_end": rows,
+            "clock_ms_mean": float(np.mean(clock_ms)), "fit_ms_mean": float(np.mean(fit_ms)),
+            "fit_ms_mean_second_half": float(np.mean(fit_ms[tail])), "fit_ms_max": float(np.max(fit_ms)),
+            "sweeps_mean": float(np.mean(sw)), "sweeps_mean_second_half": float(np.mean(sw[tail])),
+            "sweeps_max": int(np.max(sw)), "flags": int(h["flags"])}
+
+
 def main(argv=None):
     p = argparse.ArgumentParser()
     sub = p.add_subparsers(dest="cmd", required=True)
@@ -141,6 +186,10 @@ def main(argv=None):
     rc.add_argument("--workload", default=workloads.MLP4096.key, choices=list(workloads.ALL))
     rc.add_argument("--b", type=int, default=64)
     rc.add_argument("--reps", type=int, default=3)
+    pw = sub.add_parser("psw")
+    pw.add_argument("--n", type=int, default=256)
+    pw.add_argument("--iters", type=int, default=60)
+    pw.add_argument("--tol", type=float, default=1e-6)
     args = p.parse_args(argv)
     torch.cuda.set_device(0)
     if args.cmd == "aggregate":
@@ -153,6 +202,8 @@ def main(argv=None):
                 for b in sorted({0, n // 4}):
                     print(json.dumps(aggregate_case(n, d, b, args.reps)), flush=True)
                     torch.cuda.empty_cache()
+    elif args.cmd == "psw":
+        print(json.dumps(psw_case(args.n, args.iters, tol=args.tol)), flush=True)
     elif args.cmd == "received":
         print(json.dumps(received_case(args.workload, args.b, args.reps)), flush=True)
     else:

@@ -49,6 +49,22 @@ def test_state_layout_matches_c(tmp_path):
         assert int(got[f]) == getattr(dbw.DbwState, f).offset, f
 
 
+def test_psw_header_layout_matches_c(tmp_path):
+    fields = [f[0] for f in dbw.PswHeader._fields_]
+    src = tmp_path / "probe_psw.c"
+    body = "\n".join(f'printf("{f} %zu\\n", offsetof(dbw_psw_header, {f}));' for f in fields)
+    src.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "dbw.h"\nint main(void){\n'
+                   f'printf("sizeof %zu\\n", sizeof(dbw_psw_header));\n{body}\nreturn 0;}}\n')
+    exe = tmp_path / "probe_psw"
+    subprocess.run(["gcc", "-std=c99", "-I", B.INCLUDE, str(src), "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split("\n")
+    got = dict(line.split() for line in out if line)
+    assert int(got["sizeof"]) == C.sizeof(dbw.PswHeader)
+    for f in fields:
+        assert int(got[f]) == getattr(dbw.PswHeader, f).offset, f
+    assert dbw.dbw_psw_bytes(16) > 0 and dbw.dbw_psw_bytes(0) == 0 and dbw.dbw_psw_bytes(dbw.NMAX + 1) == 0
+
+
 def test_param_count_and_workspace_queries(lib):
     assert dbw.dbw_param_count([784, 10]) == 7850
     assert dbw.dbw_param_count([4096, 4096, 4096, 4096, 1000]) == 54440936
