@@ -69,15 +69,23 @@ __global__ void cast_bf16_kernel(const float* __restrict__ w, int64_t d, __nv_bf
 // blockIdx.z is a batch index (offsets batchA / batchB).
 constexpr int BM = 128, BN = 128, BK = 16;
 
-template <typename T, bool A_K, bool B_K, class Epi>
+// SPLIT (unbatched GEMMs with few output tiles): blockIdx.z is a split of K
+// instead of a batch index; split z covers k in [z * kps, (z + 1) * kps) and
+// writes its partial tile to part[z][M][N], which splitk_reduce_kernel sums in
+// split order before the epilogue.
+template <typename T, bool A_K, bool B_K, class Epi, bool SPLIT>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(int M, int N, int K, const T* __restrict__ A, int64_t lda,
                                                         int64_t batchA, const T* __restrict__ B, int64_t ldb,
-                                                        int64_t batchB, Epi epi) {
+                                                        int64_t batchB, Epi epi, int kps, float* __restrict__ part) {
     __shared__ __align__(16) float As[BK][BM];
     __shared__ __align__(16) float Bs[BK][BN];
     const int z = blockIdx.z;
-    A += (int64_t)z * batchA;
-    B += (int64_t)z * batchB;
+    if (!SPLIT) {
+        A += (int64_t)z * batchA;
+        B += (int64_t)z * batchB;
+    }
+    const int kbeg = SPLIT ? z * kps : 0;
+    const int kend = SPLIT ? (kbeg + kps < K ? kbeg + kps : K) : K;
     const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
     const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
     float acc[8][8];
@@ -86,14 +94,14 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(int M, int N, int K, con
 #pragma unroll
         for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
 
-    for (int k0 = 0; k0 < K; k0 += BK) {
+    for (int k0 = kbeg; k0 < kend; k0 += BK) {
 #pragma unroll
         for (int e = tid; e < BM * BK; e += 256) {
             int mm, kk;
             if (A_K) { mm = e / BK; kk = e % BK; } else { kk = e / BM; mm = e % BM; }
             const int gm = m0 + mm, gk = k0 + kk;
             float v = 0.f;
-            if (gm < M && gk < K) v = to_f<T>(A_K ? A[(int64_t)gm * lda + gk] : A[(int64_t)gk * lda + gm]);
+            if (gm < M && gk < kend) v = to_f<T>(A_K ? A[(int64_t)gm * lda + gk] : A[(int64_t)gk * lda + gm]);
             As[kk][mm] = v;
         }
 #pragma unroll
@@ -102,7 +110,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(int M, int N, int K, con
             if (B_K) { nn = e / BK; kk = e % BK; } else { kk = e / BN; nn = e % BN; }
             const int gn = n0 + nn, gk = k0 + kk;
             float v = 0.f;
-            if (gn < N && gk < K) v = to_f<T>(B_K ? B[(int64_t)gn * ldb + gk] : B[(int64_t)gk * ldb + gn]);
+            if (gn < N && gk < kend) v = to_f<T>(B_K ? B[(int64_t)gn * ldb + gk] : B[(int64_t)gk * ldb + gn]);
             Bs[kk][nn] = v;
         }
         __syncthreads();
@@ -128,8 +136,24 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(int M, int N, int K, con
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
             const int gn = n0 + (j < 4 ? tx * 4 + j : 64 + tx * 4 + (j - 4));
-            if (gn < N) epi(z, gm, gn, acc[i][j]);
+            if (gn < N) {
+                if (SPLIT)
+                    part[((int64_t)z * M + gm) * N + gn] = acc[i][j];
+                else
+                    epi(z, gm, gn, acc[i][j]);
+            }
         }
+    }
+}
+
+// Sum of the splits of every output element, in split order, then the epilogue.
+template <class Epi>
+__global__ void splitk_reduce_kernel(int M, int N, int splits, const float* __restrict__ part, Epi epi) {
+    const int64_t total = (int64_t)M * N;
+    for (int64_t q = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; q < total; q += (int64_t)gridDim.x * blockDim.x) {
+        float v = 0.f;
+        for (int sp = 0; sp < splits; ++sp) v += part[sp * total + q];
+        epi(0, static_cast<int>(q / N), static_cast<int>(q % N), v);
     }
 }
 
@@ -240,11 +264,37 @@ __global__ void bias_grad_kernel(const T* __restrict__ dZ, int out, int B, float
     G[(int64_t)i * ldG + offb + o] = acc;
 }
 
+// Splits of K for an unbatched GEMM with few output tiles: enough CTAs for about
+// two per SM, each split at least 4 K blocks deep; 1 = no split.
+int splitk_count(int M, int N, int K, int batch) {
+    if (batch != 1) return 1;
+    const int tiles = ((N + BN - 1) / BN) * ((M + BM - 1) / BM);
+    const int want = (2 * sm_count() + tiles - 1) / tiles;
+    const int most = K / (4 * BK);
+    int s = want < most ? want : most;
+    return s < 1 ? 1 : s;
+}
+
 template <typename T, bool A_K, bool B_K, class Epi>
 cudaError_t run_gemm(int M, int N, int K, const T* A, int64_t lda, int64_t batchA, const T* B, int64_t ldb,
-                     int64_t batchB, int batch, Epi epi, cudaStream_t st) {
+                     int64_t batchB, int batch, Epi epi, cudaStream_t st, float* split_ws = nullptr,
+                     size_t split_floats = 0) {
+    int splits = split_ws ? splitk_count(M, N, K, batch) : 1;
+    while (splits > 1 && (size_t)splits * M * N > split_floats) --splits;
+    if (splits > 1) {
+        const int kps = ((K + splits - 1) / splits + BK - 1) / BK * BK;
+        splits = (K + kps - 1) / kps;
+        dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM, splits);
+        gemm_simt_kernel<T, A_K, B_K, Epi, true><<<grid, 256, 0, st>>>(M, N, K, A, lda, 0, B, ldb, 0, epi, kps,
+                                                                       split_ws);
+        const int64_t total = (int64_t)M * N;
+        const int blocks = static_cast<int>((total + 255) / 256 < 4 * sm_count() ? (total + 255) / 256 : 4 * sm_count());
+        splitk_reduce_kernel<Epi><<<blocks, 256, 0, st>>>(M, N, splits, split_ws, epi);
+        return cudaGetLastError();
+    }
     dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM, batch);
-    gemm_simt_kernel<T, A_K, B_K, Epi><<<grid, 256, 0, st>>>(M, N, K, A, lda, batchA, B, ldb, batchB, epi);
+    gemm_simt_kernel<T, A_K, B_K, Epi, false><<<grid, 256, 0, st>>>(M, N, K, A, lda, batchA, B, ldb, batchB, epi, K,
+                                                                    nullptr);
     return cudaGetLastError();
 }
 
@@ -258,6 +308,7 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
     float* logits = reinterpret_cast<float*>(ws + P.off_logits);
     float* sloss = reinterpret_cast<float*>(ws + P.off_sloss);
     T* dz[2] = {reinterpret_cast<T*>(ws + P.off_dz[0]), reinterpret_cast<T*>(ws + P.off_dz[1])};
+    float* split_ws = P.split_floats ? reinterpret_cast<float*>(ws + P.off_split) : nullptr;
     cudaError_t e0 = cudaMemsetAsync(ws, 0, sizeof(int), st);
     if (e0 != cudaSuccess) return fail(DBW_ECUDA, "dbw_worker_grads: %s", cudaGetErrorString(e0));
     const T* wop;
@@ -284,10 +335,12 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
         const float* bias = w + P.offb[l];
         if (l < L - 1) {
             T* Aout = reinterpret_cast<T*>(ws + P.off_act[l + 1]);
-            e = run_gemm<T, true, true>(M, fout, fin, Ain, fin, 0, W, fin, 0, 1, EpiHidden<T>{bias, Aout, fout}, st);
+            e = run_gemm<T, true, true>(M, fout, fin, Ain, fin, 0, W, fin, 0, 1, EpiHidden<T>{bias, Aout, fout}, st,
+                                        split_ws, P.split_floats);
             Ain = Aout;
         } else {
-            e = run_gemm<T, true, true>(M, fout, fin, Ain, fin, 0, W, fin, 0, 1, EpiLogits{bias, logits, fout}, st);
+            e = run_gemm<T, true, true>(M, fout, fin, Ain, fin, 0, W, fin, 0, 1, EpiLogits{bias, logits, fout}, st,
+                                        split_ws, P.split_floats);
         }
         if (e != cudaSuccess) return fail(DBW_ECUDA, "forward GEMM %d: %s", l, cudaGetErrorString(e));
     }
@@ -313,7 +366,7 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
             // dZ_{l-1}[m, c] = sum_o dZ_l[m, o] W_l[o, c]: A(m, o) = dZ[m*fout + o], B(o, c) = W[o*fin + c]
             T* dnext = dz[cur ^ 1];
             e = run_gemm<T, true, false>(M, fin, fout, dZl, fout, 0, wop + P.offW[l], fin, 0, 1,
-                                         EpiDx<T>{Aprev, dnext, fin}, st);
+                                         EpiDx<T>{Aprev, dnext, fin}, st, split_ws, P.split_floats);
             if (e != cudaSuccess) return fail(DBW_ECUDA, "dX GEMM %d: %s", l, cudaGetErrorString(e));
             cur ^= 1;
         }
@@ -364,6 +417,17 @@ bool make_grads_plan(int L, const int32_t* widths, int n, int B, int prec, Grads
     P->off_dz[0] = take((size_t)M * maxw * es);
     P->off_dz[1] = take((size_t)M * maxw * es);
     P->off_wb = prec == DBW_PREC_BF16 ? take((size_t)P->d * 2) : 0;
+    // split-K scratch of the forward and input-gradient GEMMs (the largest splits x M x N)
+    size_t split = 0;
+    for (int l = 0; l < L; ++l) {
+        const int fin = widths[l], fout = widths[l + 1];
+        const size_t f = (size_t)splitk_count(P->M, fout, fin, 1) * P->M * fout;
+        const size_t x = l > 0 ? (size_t)splitk_count(P->M, fin, fout, 1) * P->M * fin : 0;
+        split = f > split ? f : split;
+        split = x > split ? x : split;
+    }
+    P->split_floats = split;
+    P->off_split = split ? take(split * 4) : 0;
     P->ws_bytes = cur;
     return true;
 }

@@ -22,6 +22,8 @@ struct GradsPlan {
     size_t off_sloss;               // [M] fp32 per-sample loss
     size_t off_dz[2];               // ping-pong dZ [M, max width] (operand type)
     size_t off_wb;                  // bf16 weights [d] (bf16 only)
+    size_t off_split;               // split-K partial tiles of the SIMT GEMMs
+    size_t split_floats;
     size_t ws_bytes;
 };
 

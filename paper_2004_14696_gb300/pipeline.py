@@ -129,6 +129,28 @@ class Iteration:
             dbw.dbw_psw_record(self.psw, wl.n, self.order, self.tsorted, self.k, stream)
             dbw.dbw_psw_estimate(self.psw, wl.n, self.T_hat, self.psw_tol, self.psw_max_sweeps, stream)
 
+    # ------------------------------------------------------------ CUDA graph
+    def capture(self, warmup=2):
+        """Record one whole iteration (on self.idx / self.times) as a CUDA graph.
+
+        Every call of the iteration is asynchronous and reads nothing back to the
+        host, so the iteration captures as is; replay() then costs one launch
+        instead of one per kernel, which is what bounds the small workloads.  The
+        inputs of each step go into self.idx / self.times before replay()."""
+        s = torch.cuda.Stream(self.device)
+        s.wait_stream(torch.cuda.current_stream(self.device))
+        with torch.cuda.stream(s):
+            for _ in range(warmup):   # first calls: lazy library setup happens outside the capture
+                self.step()
+        torch.cuda.current_stream(self.device).wait_stream(s)
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph):
+            self.step()
+        return self.graph
+
+    def replay(self):
+        self.graph.replay()
+
     # ------------------------------------------------------------ checkpoint
     def checkpoint(self):
         """Host copy of everything an iteration carries over: w and the estimator state.

@@ -5,6 +5,7 @@
     python -m paper_2004_14696_gb300.profile_case grads --workload mlp4096x3-1000_n256_B32 --reps 3
     python -m paper_2004_14696_gb300.profile_case received --workload mlp4096x3-1000_n256_B32 --b 64
     python -m paper_2004_14696_gb300.profile_case psw --n 256 --iters 60     # push-and-wait clock + Eq. (17)
+    python -m paper_2004_14696_gb300.profile_case iterate --workload mlp784-256-10_n64_B64   # whole iterations
 
 Each prints one JSON line per case with CUDA-event times (on the launching
 stream, after warm-up).  Large gradient matrices are filled on the device with
@@ -168,6 +169,47 @@ def psw_case(n, iters, seed=2004146971, model="pareto", tol=1e-6):
             "sweeps_max": int(np.max(sw)), "flags": int(h["flags"])}
 
 
+def iterate_case(key, iters, warmup, received=False, graph=False):
+    """Whole DBW iterations of a workload (the bench's step: choose b, gradients, selection,
+    aggregation, statistics; static-b workloads use their b = n/4), inputs resident on the
+    device, CUDA events around the loop.  ``graph``: each iteration is one replay of a
+    captured CUDA graph (its inputs copied into the captured buffers first)."""
+    wl = workloads.ALL[key]
+    static_b = wl.n // 4 if wl.policy == "static" else None
+    it = Iteration(wl, static_b=static_b, received=received)
+    total = warmup + iters
+    idx = torch.from_numpy(np.stack([inputs.minibatch_indices(wl.seed, t, wl.n, wl.B, wl.S)
+                                     for t in range(total)])).cuda()
+    tim = torch.from_numpy(np.stack([inputs.completion_times(wl.seed, t, wl.n, wl.time_model, **wl.time_params)
+                                     for t in range(total)])).cuda()
+    if graph:
+        it.idx.copy_(idx[0])
+        it.times.copy_(tim[0])
+        it.capture()
+
+    def one(t):
+        if graph:
+            it.idx.copy_(idx[t])
+            it.times.copy_(tim[t])
+            it.replay()
+        else:
+            it.step(idx[t], tim[t])
+    for t in range(warmup):
+        one(t)
+    st = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(st)
+    for t in range(warmup, total):
+        one(t)
+    e1.record(st)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / iters
+    return {"case": "iterate", "workload": key, "received": received, "graph": graph, "static_b": static_b,
+            "iters": iters, "ms_per_iter": ms, "iter_per_s": 1e3 / ms,
+            "status": int(it.ws[:4].view(torch.int32).item()), "launches_per_iter": it.launches_per_step()}
+
+
 def main(argv=None):
     p = argparse.ArgumentParser()
     sub = p.add_subparsers(dest="cmd", required=True)
@@ -190,6 +232,12 @@ def main(argv=None):
     pw.add_argument("--n", type=int, default=256)
     pw.add_argument("--iters", type=int, default=60)
     pw.add_argument("--tol", type=float, default=1e-6)
+    itp = sub.add_parser("iterate")
+    itp.add_argument("--workload", default=workloads.MLP784.key, choices=list(workloads.ALL))
+    itp.add_argument("--iters", type=int, default=50)
+    itp.add_argument("--warmup", type=int, default=5)
+    itp.add_argument("--received", action="store_true")
+    itp.add_argument("--graph", action="store_true", help="replay each iteration as a captured CUDA graph")
     args = p.parse_args(argv)
     torch.cuda.set_device(0)
     if args.cmd == "aggregate":
@@ -202,6 +250,9 @@ def main(argv=None):
                 for b in sorted({0, n // 4}):
                     print(json.dumps(aggregate_case(n, d, b, args.reps)), flush=True)
                     torch.cuda.empty_cache()
+    elif args.cmd == "iterate":
+        print(json.dumps(iterate_case(args.workload, args.iters, args.warmup, args.received, args.graph)),
+              flush=True)
     elif args.cmd == "psw":
         print(json.dumps(psw_case(args.n, args.iters, tol=args.tol)), flush=True)
     elif args.cmd == "received":

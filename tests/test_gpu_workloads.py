@@ -130,3 +130,38 @@ def test_checkpoint_resume_is_bit_exact_and_run_is_deterministic():
         for key in a:
             assert (a[key] == b[key]) or (a[key] != a[key] and b[key] != b[key]), key
     assert [r["t"] for r in recs] == [0, 1, 2, 3]
+
+
+@pytest.mark.parametrize("form", ["fp32", "bf16", "received", "psw"])
+def test_graph_replay_is_the_same_iteration(form):
+    """One iteration captured as a CUDA graph and replayed gives, step after step, the
+    bits eager launches give from the same state (every kernel is deterministic and
+    nothing in an iteration reads back to the host)."""
+    from paper_2004_14696_gb300.pipeline import Iteration
+    if form == "fp32":
+        wl, kw = workloads.MLP784, {}
+    else:
+        wl = workloads.Workload(key="graph_bf16", widths=(256, 128, 64, 10), n=16, B=32, prec=workloads.PREC_BF16,
+                                S=900, feature_dist="normal", time_model="pareto", time_params={"alpha": 2.0},
+                                lr=0.01, seed_offset=97)
+        kw = {"received": form == "received", "clock": "psw" if form == "psw" else "psi"}
+    eager = Iteration(wl, **kw)
+    graphed = Iteration(wl, **kw)
+    graphed.load_inputs(0)
+    ck = eager.checkpoint()
+    graphed.capture()              # its warm-up steps moved graphed's state: restart both from ck
+    graphed.restore(ck)
+    if form == "psw":
+        dbw.dbw_psw_init(graphed.psw, wl.n)
+        graphed.T_hat.fill_(float("nan"))
+    for t in range(5):
+        eager.load_inputs(t)
+        eager.step()
+        graphed.load_inputs(t)
+        graphed.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(eager.w, graphed.w), t
+        assert torch.equal(eager.stats.view(torch.int64), graphed.stats.view(torch.int64)), t
+        assert torch.equal(eager.b, graphed.b) and torch.equal(eager.mask, graphed.mask), t
+        if form == "psw":
+            assert torch.equal(eager.psw, graphed.psw), t
