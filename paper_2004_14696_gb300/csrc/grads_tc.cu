@@ -26,27 +26,95 @@ namespace {
 
 inline int64_t rup(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 
-// W_l [out, in] fp32 (rows of length in) -> wb [out, ldw] bf16 and wt [in, ldwt] bf16.
-__global__ void cast_transpose_kernel(const float* __restrict__ W, int out, int in, __nv_bfloat16* __restrict__ wb,
-                                      int64_t ldw, __nv_bfloat16* __restrict__ wt, int64_t ldwt) {
-    __shared__ __nv_bfloat16 tile[32][33];
-    const int i0 = blockIdx.x * 32, o0 = blockIdx.y * 32;
-    const int tx = threadIdx.x, ty = threadIdx.y;   // 32 x 8
-    for (int r = ty; r < 32; r += 8) {
-        const int o = o0 + r, i = i0 + tx;
-        __nv_bfloat16 v = __float2bfloat16_rn(0.f);
-        if (o < out && i < in) {
-            v = __float2bfloat16_rn(W[static_cast<int64_t>(o) * in + i]);
-            wb[static_cast<int64_t>(o) * ldw + i] = v;
+// One pass over fp32 rows: out[m, :] = bf16(src[row(m), :]) and outT = its
+// transpose, for m < rows (cols logical columns; padding is never written).  A
+// CTA handles a 64 x 64 tile: the rows are read as float4 where aligned, the
+// bf16 tile is written row-major with 8-byte stores and, through a padded
+// shared-memory tile, column-major with 8-byte stores along m.  row(m) < 0 makes
+// row m zero.  Used for X (gathered minibatch rows) and for W_l (rows = out).
+template <class RowMap>
+__global__ void __launch_bounds__(256) cast_transpose_tile_kernel(const float* __restrict__ src, int64_t lds,
+                                                                  int rows, int cols, RowMap rowmap,
+                                                                  __nv_bfloat16* __restrict__ out, int64_t ldo,
+                                                                  __nv_bfloat16* __restrict__ outT, int64_t ldT) {
+    __shared__ __nv_bfloat16 tile[64][64 + 8];
+    const int c0 = blockIdx.x * 64, m0 = blockIdx.y * 64;
+    const int live = rowmap.live(rows);
+    if (m0 >= live) return;
+    const int t = threadIdx.x;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int e = t + 256 * q;
+        const int r = e >> 4, c = c0 + 4 * (e & 15);
+        const int m = m0 + r;
+        float v[4] = {0.f, 0.f, 0.f, 0.f};
+        if (m < live && c < cols) {
+            const int64_t sr = rowmap(m);
+            if (sr >= 0) {
+                const float* p = src + sr * lds + c;
+                if (c + 3 < cols && ((reinterpret_cast<uintptr_t>(p) & 15u) == 0)) {
+                    const float4 f = *reinterpret_cast<const float4*>(p);
+                    v[0] = f.x, v[1] = f.y, v[2] = f.z, v[3] = f.w;
+                } else {
+                    for (int j = 0; j < 4 && c + j < cols; ++j) v[j] = p[j];
+                }
+            }
         }
-        tile[r][tx] = v;
+        __nv_bfloat16 h[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) h[j] = __float2bfloat16_rn(v[j]);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) tile[r][4 * (e & 15) + j] = h[j];
+        if (m < live && c < cols) {
+            __nv_bfloat16* o = out + static_cast<int64_t>(m) * ldo + c;
+            if (c + 3 < cols && ((reinterpret_cast<uintptr_t>(o) & 7u) == 0)) {
+                uint2 pk;
+                pk.x = static_cast<uint32_t>(__bfloat16_as_ushort(h[0])) |
+                       (static_cast<uint32_t>(__bfloat16_as_ushort(h[1])) << 16);
+                pk.y = static_cast<uint32_t>(__bfloat16_as_ushort(h[2])) |
+                       (static_cast<uint32_t>(__bfloat16_as_ushort(h[3])) << 16);
+                *reinterpret_cast<uint2*>(o) = pk;
+            } else {
+                for (int j = 0; j < 4 && c + j < cols; ++j) o[j] = h[j];
+            }
+        }
     }
     __syncthreads();
-    for (int r = ty; r < 32; r += 8) {
-        const int i = i0 + r, o = o0 + tx;
-        if (i < in && o < out) wt[static_cast<int64_t>(i) * ldwt + o] = tile[tx][r];
+    if (!outT) return;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int e = t + 256 * q;
+        const int cc = e >> 4, r = 4 * (e & 15);
+        const int c = c0 + cc, m = m0 + r;
+        if (c >= cols || m >= live) continue;
+        __nv_bfloat16* o = outT + static_cast<int64_t>(c) * ldT + m;
+        if (m + 3 < live && ((reinterpret_cast<uintptr_t>(o) & 7u) == 0)) {
+            uint2 pk;
+            pk.x = static_cast<uint32_t>(__bfloat16_as_ushort(tile[r][cc])) |
+                   (static_cast<uint32_t>(__bfloat16_as_ushort(tile[r + 1][cc])) << 16);
+            pk.y = static_cast<uint32_t>(__bfloat16_as_ushort(tile[r + 2][cc])) |
+                   (static_cast<uint32_t>(__bfloat16_as_ushort(tile[r + 3][cc])) << 16);
+            *reinterpret_cast<uint2*>(o) = pk;
+        } else {
+            for (int j = 0; j < 4 && m + j < live; ++j) o[j] = tile[r + j][cc];
+        }
     }
 }
+
+// Row maps of cast_transpose_tile_kernel.
+struct IdentityRows {   // W_l: row o of the matrix
+    __device__ int live(int rows) const { return rows; }
+    __device__ int64_t operator()(int m) const { return m; }
+};
+struct GatherRows {     // X of the per-worker pass: pool row idx[m]; an index outside [0, S) reads row 0
+    const int32_t* idx;
+    int64_t S;
+    __device__ int live(int rows) const { return rows; }
+    __device__ int64_t operator()(int m) const {
+        const int64_t r = idx[m];
+        return (r < 0 || r >= S) ? 0 : r;
+    }
+};
 
 // Rows of the stacked buffers that a received-workers pass computes: the k B
 // received rows rounded up to the 128-row GEMM tile (all M when kdev is null).
@@ -56,6 +124,24 @@ __device__ __forceinline__ int live_rows(const int* kdev, int B, int M) {
     const long long r = (static_cast<long long>(k > 0 ? k : 0) * B + 127) / 128 * 128;
     return r < M ? static_cast<int>(r) : M;
 }
+
+// X of the received-workers pass: row m of slot s = m / B < k is pool row
+// idx[sel[s] B + m % B] (an index outside [0, S) reads row 0); rows from k B up to
+// the live row count are zero; later rows are not written.
+struct ReceivedRows {
+    const int32_t* idx;
+    const int32_t* sel;
+    const int* kdev;
+    int B;
+    int64_t S;
+    __device__ int live(int rows) const { return live_rows(kdev, B, rows); }
+    __device__ int64_t operator()(int m) const {
+        const int s = m / B;
+        if (s >= *kdev) return -1;
+        const int64_t r = idx[static_cast<int64_t>(sel[s]) * B + (m - s * B)];
+        return (r < 0 || r >= S) ? 0 : r;
+    }
+};
 
 // dst [cols, ldd] = src [rows, lds]^T  (bf16), rows x cols logical; with kdev, only
 // the live rows (live_rows) are transposed.
@@ -78,30 +164,6 @@ __global__ void transpose_bf16_kernel(const __nv_bfloat16* __restrict__ src, int
     }
 }
 
-// X[m, :] = bf16(pool[idx[m], :]); an index outside [0, S) reads row 0 (the loss
-// kernel poisons that worker).
-__global__ void gather_bf16_kernel(const float* __restrict__ pool, int64_t S, int in, const int32_t* __restrict__ idx,
-                                   int M, __nv_bfloat16* __restrict__ X, int64_t ldx) {
-    for (int m = blockIdx.y; m < M; m += gridDim.y) {
-        int64_t r = idx[m];
-        if (r < 0 || r >= S) r = 0;
-        const float* src = pool + r * in;
-        __nv_bfloat16* dst = X + static_cast<int64_t>(m) * ldx;
-        for (int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4; c < in; c += gridDim.x * blockDim.x * 4) {
-            const float4 v = *reinterpret_cast<const float4*>(src + c);
-            __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
-            if (c + 3 < in) {
-                *reinterpret_cast<__nv_bfloat162*>(dst + c) = a;
-                *reinterpret_cast<__nv_bfloat162*>(dst + c + 2) = b;
-            } else {
-                for (int e = c; e < in; ++e) dst[e] = __float2bfloat16_rn(src[e]);
-            }
-        }
-    }
-}
-
-// Per worker (one CTA): stable log-softmax cross entropy per sample, dZ = (softmax - onehot) / B
-// as bf16 into dZ [M, ldz], worker loss = mean of its B sample losses (sample order).
 // With ``sel`` (received-workers pass): CTA s handles slot s, i.e. worker sel[s]
 // (stacked rows s B .., samples idx[sel[s] B + r], loss[sel[s]]); slots s >= k
 // zero their dZ rows up to the live row count and stop.
@@ -197,37 +259,6 @@ __global__ void __launch_bounds__(1024) compact_received_kernel(const uint8_t* _
         int k = 0;
         for (int q = 0; q < 32; ++q) k += warp_tot[q];
         *kout = k;
-    }
-}
-
-// X[m, :] = bf16(pool[idx[sel[s] B + r], :]) for m = s B + r, s < k; live rows past
-// k B are zeroed (so every stacked row a GEMM tile reads is finite).
-__global__ void gather_received_kernel(const float* __restrict__ pool, int64_t S, int in,
-                                       const int32_t* __restrict__ idx, const int32_t* __restrict__ sel,
-                                       const int* __restrict__ kdev, int B, int M, __nv_bfloat16* __restrict__ X,
-                                       int64_t ldx) {
-    const int k = *kdev;
-    const int live = live_rows(kdev, B, M);
-    for (int m = blockIdx.y; m < live; m += gridDim.y) {
-        const int s = m / B;
-        __nv_bfloat16* dst = X + static_cast<int64_t>(m) * ldx;
-        if (s >= k) {
-            for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < in; c += gridDim.x * blockDim.x)
-                dst[c] = __float2bfloat16_rn(0.f);
-            continue;
-        }
-        int64_t r = idx[static_cast<int64_t>(sel[s]) * B + (m - s * B)];
-        if (r < 0 || r >= S) r = 0;   // the loss kernel poisons that worker
-        const float* src = pool + r * in;
-        for (int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4; c < in; c += gridDim.x * blockDim.x * 4) {
-            const float4 v = *reinterpret_cast<const float4*>(src + c);
-            if (c + 3 < in) {
-                *reinterpret_cast<__nv_bfloat162*>(dst + c) = __floats2bfloat162_rn(v.x, v.y);
-                *reinterpret_cast<__nv_bfloat162*>(dst + c + 2) = __floats2bfloat162_rn(v.z, v.w);
-            } else {
-                for (int e = c; e < in; ++e) dst[e] = __float2bfloat16_rn(src[e]);
-            }
-        }
     }
 }
 
@@ -394,18 +425,16 @@ int worker_grads_tc(const TcPlan& P, const float* w, const float* pool, int64_t 
     // bf16 weights and their transposes
     for (int l = 0; l < L; ++l) {
         const int fin = g.widths[l], fout = g.widths[l + 1];
-        dim3 grid((fin + 31) / 32, (fout + 31) / 32);
-        cast_transpose_kernel<<<grid, dim3(32, 8), 0, st>>>(w + g.offW[l], fout, fin, bf(P.off_wb[l]), P.ldw[l],
-                                                            bf(P.off_wt[l]), P.ldwt[l]);
+        dim3 grid((fin + 63) / 64, (fout + 63) / 64);
+        cast_transpose_tile_kernel<<<grid, 256, 0, st>>>(w + g.offW[l], fin, fout, fin, IdentityRows{},
+                                                         bf(P.off_wb[l]), P.ldw[l], bf(P.off_wt[l]), P.ldwt[l]);
     }
     // X and X^T
     {
         const int in = g.widths[0];
-        dim3 grid((in + 1023) / 1024, M < 65535 ? M : 65535);
-        gather_bf16_kernel<<<grid, 256, 0, st>>>(pool, S, in, idx, M, bf(P.off_act[0]), P.ldact[0]);
-        dim3 tg((in + 31) / 32, (M + 31) / 32);
-        transpose_bf16_kernel<<<tg, dim3(32, 8), 0, st>>>(bf(P.off_act[0]), M, in, P.ldact[0], bf(P.off_actT[0]),
-                                                          P.M8);
+        dim3 grid((in + 63) / 64, (M + 63) / 64);
+        cast_transpose_tile_kernel<<<grid, 256, 0, st>>>(pool, in, M, in, GatherRows{idx, S}, bf(P.off_act[0]),
+                                                         P.ldact[0], bf(P.off_actT[0]), P.M8);
     }
     e = cudaGetLastError();
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_worker_grads: %s", cudaGetErrorString(e));
@@ -534,17 +563,15 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
     compact_received_kernel<<<1, 1024, 0, st>>>(mask, n, sel, kdev, loss);
     for (int l = 0; l < L; ++l) {
         const int fin = g.widths[l], fout = g.widths[l + 1];
-        dim3 grid((fin + 31) / 32, (fout + 31) / 32);
-        cast_transpose_kernel<<<grid, dim3(32, 8), 0, st>>>(w + g.offW[l], fout, fin, bf(T.off_wb[l]), T.ldw[l],
-                                                            bf(T.off_wt[l]), T.ldwt[l]);
+        dim3 grid((fin + 63) / 64, (fout + 63) / 64);
+        cast_transpose_tile_kernel<<<grid, 256, 0, st>>>(w + g.offW[l], fin, fout, fin, IdentityRows{},
+                                                         bf(T.off_wb[l]), T.ldw[l], bf(T.off_wt[l]), T.ldwt[l]);
     }
     {
         const int in = g.widths[0];
-        dim3 grid((in + 1023) / 1024, M < 65535 ? M : 65535);
-        gather_received_kernel<<<grid, 256, 0, st>>>(pool, S, in, idx, sel, kdev, B, M, bf(T.off_act[0]), T.ldact[0]);
-        dim3 tg((in + 31) / 32, (M + 31) / 32);
-        transpose_bf16_kernel<<<tg, dim3(32, 8), 0, st>>>(bf(T.off_act[0]), M, in, T.ldact[0], bf(T.off_actT[0]),
-                                                          T.M8, kdev, B);
+        dim3 grid((in + 63) / 64, (M + 63) / 64);
+        cast_transpose_tile_kernel<<<grid, 256, 0, st>>>(pool, in, M, in, ReceivedRows{idx, sel, kdev, B, S},
+                                                         bf(T.off_act[0]), T.ldact[0], bf(T.off_actT[0]), T.M8);
     }
     e = cudaGetLastError();
     if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));

@@ -190,22 +190,24 @@ class Iteration:
         return rec
 
     def launches_per_step(self):
-        """Kernels libdbw launches per step (for the bench's launch count)."""
+        """Kernels libdbw launches per step (for the bench's launch count); the status-word
+        memsets are copies, not kernels.  On the fp32 SIMT path a split-K GEMM adds one
+        reduce kernel, which this count leaves out."""
         L = len(self.wl.widths) - 1
         choose = (0 if self.static_b is not None else 1) + (3 if self.clock == "psw" else 0)   # + arrivals, record, fit
         if self.received:
-            # select; status memset, compaction, L weight cast-transposes, gather + X^T, L forward
-            # GEMMs, loss + dZ^T, per layer (mean-gradient GEMM, bias sums, bias update, Gram),
-            # L-1 dX GEMMs, finish; grad_stats (2)
-            return choose + 1 + (1 + 1 + L + 2 + L + 2 + 4 * L + (L - 1) + 1) + 2
+            # select; compaction, L weight cast-transposes, X and X^T, L forward GEMMs, loss + dZ^T,
+            # per layer (mean-gradient GEMM, bias sums, bias update, Gram), L-1 dX GEMMs, finish;
+            # grad_stats (2)
+            return choose + 1 + (1 + L + 1 + L + 2 + 4 * L + (L - 1) + 1) + 2
         if self.wl.prec == dbw.PREC_BF16 and self.wl.B % 32 == 0:
-            # tcgen05 pass: status memset, L weight cast-transposes, gather + X^T, L forward
-            # GEMMs, loss + dZ^T, L dW GEMMs, L bias gradients, L-1 dX GEMMs
-            grads = 1 + L + 2 + L + 2 + L + L + (L - 1)
+            # tcgen05 pass: L weight cast-transposes, X and X^T, L forward GEMMs, loss + dZ^T,
+            # L dW GEMMs, L bias gradients, L-1 dX GEMMs
+            grads = L + 1 + L + 2 + L + L + (L - 1)
         else:
-            grads = 1 + 1 + L + 1 + L + L + (L - 1)    # status memset, gather, fwd, loss, dW, bias, dX
+            grads = 1 + L + 1 + L + L + (L - 1)    # gather, forward, loss, dW, bias, dX
             if self.wl.prec == dbw.PREC_BF16:
-                grads += 1                              # bf16 weight cast
+                grads += 1                          # bf16 weight cast
         return choose + grads + 1 + 1 + 2
 
 

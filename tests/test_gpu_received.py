@@ -38,6 +38,9 @@ RX_B32 = _wl("rx_b32", (256, 128, 64, 10), 8, 32, 91)
 RX_B64 = _wl("rx_b64", (300, 200, 100, 7), 5, 64, 92, "uniform")
 RX_B128 = _wl("rx_b128", (128, 96, 10), 3, 128, 93)
 RX_B256 = _wl("rx_b256", (200, 64, 12), 3, 256, 94)
+# k B long enough for the mean-gradient GEMM to split K over several work items (its
+# outputs have far fewer tiles than SMs); b = 31 leaves one worker, so most splits are empty
+RX_SPLIT = _wl("rx_split", (256, 96, 10), 32, 64, 96)
 
 
 def slot_rows(mask, B):
@@ -106,7 +109,7 @@ def check_against_oracle(it, wl, w0, idx, times, b, workers=None):
 
 
 @pytest.mark.parametrize("wl,b", [(RX_B32, 0), (RX_B32, 3), (RX_B32, 7), (RX_B64, 0), (RX_B64, 2),
-                                  (RX_B128, 1), (RX_B256, 0), (RX_B256, 2)],
+                                  (RX_B128, 1), (RX_B256, 0), (RX_B256, 2), (RX_SPLIT, 5), (RX_SPLIT, 31)],
                          ids=lambda v: v.key if hasattr(v, "key") else f"b{v}")
 def test_received_iteration_matches_oracle(wl, b):
     """All outputs of one received-workers iteration against the oracle: loss (NaN for
