@@ -59,10 +59,10 @@ struct RxPlan {
     int CT;                            // Gram column tiles per 128-row tile: max(1, B / 128)
     size_t off_sel;                    // int32 [n]: received workers, increasing
     size_t off_k;                      // int32: k
-    size_t off_csum;                   // fp32 [n, max out]: per-slot bias gradient sums
+    size_t off_bpart;                  // fp32 [ceil(M / 256), max out]: bias column sums per 256-row chunk
     size_t off_pw[DBW_LMAX];           // fp64 [tiles_l * 4]: pieces of ||g_t(W_l)||^2
     int64_t npw[DBW_LMAX];
-    size_t off_pb[DBW_LMAX];           // fp64 [ceil(out_l / 128)]: pieces of ||g_t(b_l)||^2
+    size_t off_pb[DBW_LMAX];           // fp64 [ceil(out_l / 256)]: pieces of ||g_t(b_l)||^2
     int npb[DBW_LMAX];
     size_t off_pg[DBW_LMAX];           // fp64 [(M / 32) * CT]: Gram pieces of ||g_j||^2
     size_t ws_bytes;

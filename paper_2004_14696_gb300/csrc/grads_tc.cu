@@ -262,45 +262,73 @@ __global__ void __launch_bounds__(1024) compact_received_kernel(const uint8_t* _
     }
 }
 
-// csum[s * out + o] = sum_{r < B} dZ[s B + r, o] (rows in order) for slots s < k:
-// worker sel[s]'s bias gradient, the same sums the per-worker pass writes into G.
-__global__ void slot_colsum_kernel(const __nv_bfloat16* __restrict__ dZ, int64_t ldz, int out, int B,
-                                   const int* __restrict__ kdev, float* __restrict__ csum) {
-    const int s = blockIdx.y;
-    const int o = blockIdx.x * blockDim.x + threadIdx.x;
-    if (s >= *kdev || o >= out) return;
-    const __nv_bfloat16* p = dZ + static_cast<int64_t>(s) * B * ldz + o;
-    float acc = 0.f;
-    for (int r = 0; r < B; ++r) acc += __bfloat162float(p[static_cast<int64_t>(r) * ldz]);
-    csum[static_cast<int64_t>(s) * out + o] = acc;
+// Bias part of Eqs. (3)-(4), g[o] = (1/k) sum_{r < k B} dZ[r, o], in two steps.
+// bias_rows_kernel: one CTA per (256 columns, 256-row chunk); thread (warp y, lane)
+// sums 8 columns (16-byte loads) over rows y, y + 8, ... of the chunk, and the 8
+// warps' sums are added in warp order into part[chunk][o].  Chunks past k B write
+// nothing.
+__global__ void __launch_bounds__(256) bias_rows_kernel(const __nv_bfloat16* __restrict__ dZ, int64_t ldz, int out,
+                                                        int B, const int* __restrict__ kdev, float* __restrict__ part) {
+    __shared__ float red[8][256];
+    const int k = *kdev;
+    const int rows = k > 0 ? k * B : 0;
+    const int r0 = blockIdx.y * 256;
+    if (r0 >= rows) return;
+    const int lane = threadIdx.x & 31, y = threadIdx.x >> 5;
+    const int c = blockIdx.x * 256 + 8 * lane;
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    const int rend = r0 + 256 < rows ? r0 + 256 : rows;
+    if (c + 7 < out) {
+#pragma unroll 4
+        for (int r = r0 + y; r < rend; r += 8) {
+            const uint4 raw = *reinterpret_cast<const uint4*>(dZ + static_cast<int64_t>(r) * ldz + c);
+            const __nv_bfloat16* h = reinterpret_cast<const __nv_bfloat16*>(&raw);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) acc[j] += __bfloat162float(h[j]);
+        }
+    } else {
+        for (int r = r0 + y; r < rend; r += 8)
+            for (int j = 0; j < 8 && c + j < out; ++j) acc[j] += __bfloat162float(dZ[static_cast<int64_t>(r) * ldz + c + j]);
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) red[y][8 * lane + j] = acc[j];
+    __syncthreads();
+    const int o = blockIdx.x * 256 + threadIdx.x;
+    if (o < out) {
+        float t = 0.f;
+        for (int q = 0; q < 8; ++q) t += red[q][threadIdx.x];
+        part[static_cast<int64_t>(blockIdx.y) * out + o] = t;
+    }
 }
 
-// Bias part of Eqs. (3)-(4): g = (1/k) sum_{s < k} csum[s, o] (slots in order),
-// wb[o] -= lr g, gb[o] = g (nullable); the CTA's sum of g^2 (fp64, fixed tree)
-// into pieces[blockIdx.x].
-__global__ void __launch_bounds__(128) bias_mean_update_kernel(const float* __restrict__ csum, int out,
+// bias_mean_update_kernel: g[o] = (1/k) sum of the chunks' sums (chunk order),
+// wb[o] -= lr g, gb[o] = g (nullable); the CTA's sum of g^2 (fp64, fixed tree) into
+// pieces[blockIdx.x].
+__global__ void __launch_bounds__(256) bias_mean_update_kernel(const float* __restrict__ part, int out, int B,
                                                                const int* __restrict__ kdev, float lr,
                                                                float* __restrict__ wb, float* __restrict__ gb,
                                                                double* __restrict__ pieces) {
-    __shared__ double red[128];
+    __shared__ double red[8];
     const int k = *kdev;
-    const int o = blockIdx.x * blockDim.x + threadIdx.x;
+    const int chunks = k > 0 ? (k * B + 255) / 256 : 0;
+    const int o = blockIdx.x * 256 + threadIdx.x;
     double sq = 0.0;
     if (o < out && k > 0) {
-        float acc = 0.f;
-        for (int s = 0; s < k; ++s) acc += csum[static_cast<int64_t>(s) * out + o];
-        const float g = acc * (1.0f / static_cast<float>(k));
+        float t = 0.f;
+        for (int q = 0; q < chunks; ++q) t += part[static_cast<int64_t>(q) * out + o];
+        const float g = t * (1.0f / static_cast<float>(k));
         wb[o] = fmaf(-lr, g, wb[o]);
         if (gb) gb[o] = g;
         sq = static_cast<double>(g) * g;
     }
-    red[threadIdx.x] = sq;
+    for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = sq;
     __syncthreads();
-    for (int h = 64; h > 0; h >>= 1) {
-        if (threadIdx.x < h) red[threadIdx.x] += red[threadIdx.x + h];
-        __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < 8; ++w) t += red[w];
+        pieces[blockIdx.x] = t;
     }
-    if (threadIdx.x == 0) pieces[blockIdx.x] = red[0];
 }
 
 struct FinishArgs {
@@ -527,16 +555,16 @@ bool make_rx_plan(int L, const int32_t* widths, int n, int B, RxPlan* P) {
         cur += (bytes + 255) / 256 * 256;
         return at;
     };
-    int maxout = 0;
-    for (int l = 0; l < L; ++l) maxout = g.widths[l + 1] > maxout ? g.widths[l + 1] : maxout;
     P->off_sel = take(static_cast<size_t>(n) * 4);
     P->off_k = take(4);
-    P->off_csum = take(static_cast<size_t>(n) * maxout * 4);
+    int maxout = 0;
+    for (int l = 0; l < L; ++l) maxout = g.widths[l + 1] > maxout ? g.widths[l + 1] : maxout;
+    P->off_bpart = take(static_cast<size_t>((g.M + 255) / 256) * maxout * 4);
     for (int l = 0; l < L; ++l) {
         const int fin = g.widths[l], fout = g.widths[l + 1];
         P->npw[l] = static_cast<int64_t>((fout + 127) / 128) * ((fin + 255) / 256) * 4;
         P->off_pw[l] = take(static_cast<size_t>(P->npw[l]) * 8);
-        P->npb[l] = (fout + 127) / 128;
+        P->npb[l] = (fout + 255) / 256;
         P->off_pb[l] = take(static_cast<size_t>(P->npb[l]) * 8);
         P->off_pg[l] = take(static_cast<size_t>(g.M / 32) * P->CT * 8);
     }
@@ -553,7 +581,7 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
     int* status = reinterpret_cast<int*>(ws + T.off_status);
     int32_t* sel = reinterpret_cast<int32_t*>(ws + P.off_sel);
     int* kdev = reinterpret_cast<int*>(ws + P.off_k);
-    float* csum = reinterpret_cast<float*>(ws + P.off_csum);
+    float* bpart = reinterpret_cast<float*>(ws + P.off_bpart);
     auto bf = [&](size_t off) { return reinterpret_cast<__nv_bfloat16*>(ws + off); };
     auto f64 = [&](size_t off) { return reinterpret_cast<double*>(ws + off); };
     const char* what = "dbw_received_grads_update";
@@ -628,9 +656,9 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
         int rc = tc_gemm(TC_GBAR, bf(T.off_dzT), T.M8, fout, M, bf(T.off_actT[l]), T.M8, fin, M, fout, fin, M, 1, 0,
                          gb, status, st);
         if (rc) return rc;
-        slot_colsum_kernel<<<dim3((fout + 127) / 128, n), 128, 0, st>>>(bf(T.off_dz[cur]), T.ldz, fout, B, kdev,
-                                                                         csum);
-        bias_mean_update_kernel<<<P.npb[l], 128, 0, st>>>(csum, fout, kdev, lr, w + g.offb[l],
+        bias_rows_kernel<<<dim3((fout + 255) / 256, (M + 255) / 256), 256, 0, st>>>(bf(T.off_dz[cur]), T.ldz, fout,
+                                                                                   B, kdev, bpart);
+        bias_mean_update_kernel<<<P.npb[l], 256, 0, st>>>(bpart, fout, B, kdev, lr, w + g.offb[l],
                                                            gbar ? gbar + g.offb[l] : nullptr, f64(P.off_pb[l]));
         e = cudaGetLastError();
         if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
