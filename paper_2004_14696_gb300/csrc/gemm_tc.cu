@@ -667,10 +667,14 @@ cudaError_t launch_dw(const CUtensorMap& a, const CUtensorMap& b, int Mr, int Nr
     return cudaGetLastError();
 }
 
+#ifndef DBW_PERSISTENT_STAGES
+#define DBW_PERSISTENT_STAGES 4   // TMA ring depth of the persistent GEMM (48 KB per stage)
+#endif
+
 template <int KIND>
 cudaError_t launch_persistent(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, const TcEpi& e,
                               int* status, cudaStream_t st) {
-    constexpr int STAGES = 4;
+    constexpr int STAGES = DBW_PERSISTENT_STAGES;
     using Cfg = TcCfg<256, 64, STAGES>;
     auto kern = tc_gemm_persistent_kernel<KIND, STAGES>;
     cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
