@@ -264,6 +264,7 @@ def _run_dbw(args, rank, world, local_rank, clk):
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     dbw.dbw_profile_dw(True)
+    dbw.dbw_profile_gemm(True)
     wall0 = time.time()
     t_start.record(stream)
     for t in range(W, total):
@@ -274,6 +275,8 @@ def _run_dbw(args, rank, world, local_rank, clk):
     time.sleep(0.15)                # let the sampler deliver the samples of the window
     dw_ms, dw_launches, dw_bytes = dbw.dbw_profile_dw_read()
     dbw.dbw_profile_dw(False)
+    gm_ms, gm_launches = dbw.dbw_profile_gemm_read()
+    dbw.dbw_profile_gemm(False)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
@@ -347,12 +350,25 @@ def _run_dbw(args, rank, world, local_rank, clk):
     ms_step = elapsed_ms / K
     value = job_value(world, K, elapsed_ms)
     gemm_flop = 0
+    tc_flop = 0
     wd = wl.widths
     M = n * B
     for l in range(len(wd) - 1):
         gemm_flop += 2 * M * wd[l] * wd[l + 1] * 2          # forward + per-worker dW
+        tc_flop += 2 * M * wd[l] * wd[l + 1]                # forward
         if l > 0:
             gemm_flop += 2 * M * wd[l] * wd[l + 1]          # input gradient
+            tc_flop += 2 * M * wd[l] * wd[l + 1]
+    # the forward and input-gradient GEMMs (persistent tcgen05 kernel), timed live
+    tensor = None
+    if gm_launches:
+        tf = tc_flop * K / (gm_ms * 1e-3) / 1e12
+        tensor = {"kernel": "tc_gemm_persistent_kernel (forward + input-gradient GEMMs, in dbw_worker_grads)",
+                  "bound": "tensor", "achieved": tf, "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s",
+                  "frac": tf / pk["bf16_tflops_sustained"], "traffic": None,
+                  "algorithmic_flop_per_step": tc_flop, "ms_per_step": gm_ms / K,
+                  "launches_timed": gm_launches, "share_of_step": gm_ms / elapsed_ms,
+                  "peak_kind": "bf16 dense, sustained", "peak_source": pk["source"]}
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
         "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
@@ -366,6 +382,7 @@ def _run_dbw(args, rank, world, local_rank, clk):
                                "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
                                "frac": achieved / pk["hbm_gbs"], "traffic": traffic,
                                "algorithmic_bytes_per_launch": agg_bytes, "peak_source": pk["source"]},
+        "roofline_tensor": tensor,
         "phases_ms": phase_ms,
         "gemm": {"flop_per_step": gemm_flop, "worker_grads_tflops": gemm_flop / (phase_ms["worker_grads"] * 1e-3) / 1e12},
         "gpu_launches": None,
@@ -384,6 +401,16 @@ def _run_dbw(args, rank, world, local_rank, clk):
                         "frac_of_sustained": flop / t_upd / 1e12 / pk["bf16_tflops_sustained"]
                         if pk.get("bf16_tflops_sustained") else None,
                         "peak_sustained": pk.get("bf16_tflops_sustained"), "peak_source": pk["source"]}
+        gms, gl = rx.pop("_gemm")
+        if gl:
+            tf = flop / (gms * 1e-3) / 1e12
+            rx["roofline"] = {"kernel": "tc_gemm_persistent_kernel (forward, mean-gradient and input-gradient "
+                                        "GEMMs, in dbw_received_grads_update)",
+                              "bound": "tensor", "achieved": tf, "peak": pk["bf16_tflops_sustained"],
+                              "unit": "TFLOP/s", "frac": tf / pk["bf16_tflops_sustained"], "traffic": None,
+                              "algorithmic_flop_per_step": flop, "ms_per_step": gms, "launches_timed": gl * K,
+                              "share_of_step": gms / rx["ms_per_step"], "peak_kind": "bf16 dense, sustained",
+                              "peak_source": pk["source"]}
         out["received_form"] = rx
     return out
 
@@ -433,11 +460,14 @@ def _time_received(wl, dev, idx_d, tim_d, W, K, stream, world):
         dist.barrier()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
+    dbw.dbw_profile_gemm(True)
     t0.record(stream)
     for t in range(W, total):
         one(t, True)
     t1.record(stream)
     torch.cuda.synchronize(dev)
+    gm_ms, gm_launches = dbw.dbw_profile_gemm_read()
+    dbw.dbw_profile_gemm(False)
     ms = t0.elapsed_time(t1)
     (ms,) = combine_over_ranks([ms], world, dev)
     phase = {nm: sum(ev[t][i].elapsed_time(ev[t][i + 1]) for t in range(W, total)) / K for i, nm in enumerate(names)}
@@ -445,7 +475,8 @@ def _time_received(wl, dev, idx_d, tim_d, W, K, stream, world):
     status = int(it.ws[:4].view(torch.int32).item())
     out = {"call": "dbw_received_grads_update", "value": job_value(world, K, ms), "unit": UNIT,
            "ms_per_step": ms / K, "phases_ms": phase, "mean_k": float(kv.mean()), "device_status": status,
-           "gpu_launches": it.launches_per_step() * K, "_k": float(kv.mean())}
+           "gpu_launches": it.launches_per_step() * K, "_k": float(kv.mean()),
+           "_gemm": (gm_ms / K, gm_launches // K)}
     del it
     torch.cuda.empty_cache()
     return out

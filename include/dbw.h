@@ -189,6 +189,20 @@ int dbw_profile_dw(int enable);
 int dbw_profile_dw_read(double* total_ms, int64_t* launches, double* total_bytes);
 
 /*
+ * Opt-in timing of the persistent tensor-core GEMMs: the forward GEMMs of every
+ * layer and the input-gradient GEMMs inside dbw_worker_grads (bf16 models), and
+ * in dbw_received_grads_update also the mean-gradient GEMM of every layer.  Each
+ * such launch is bracketed by CUDA events on the call's stream while enabled.
+ * dbw_profile_gemm(enable) turns it on or off and forgets earlier records;
+ * dbw_profile_gemm_read waits for the recorded events and returns the summed
+ * launch durations (ms) and the number of launches, then forgets them.  The
+ * caller knows the flops: in the received form M (or K) is k*B with k read on
+ * the device.  Host only; not for use during stream capture.
+ */
+int dbw_profile_gemm(int enable);
+int dbw_profile_gemm_read(double* total_ms, int64_t* launches);
+
+/*
  * Eq. (4): the PS waits for the first k = n - b gradients.
  * Arrival order is (times[i], i) ascending (ties go to the lower worker index).
  *

@@ -751,26 +751,27 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
         const int bk = (K % 64 == 0) ? 64 : 32;
         // algorithmic bytes: G written once (fp32), both bf16 operands read once
         const double dw_bytes = 4.0 * batch * double(M) * N + 2.0 * batch * double(K) * (double(M) + N);
-        void* prof = dw_profile_begin(st, dw_bytes);
         if (!tc_make_map(&ta, A, rowsA, colsA, lda, bk, BM) || !tc_make_map(&tb, B, rowsB, colsB, ldb, bk, DW_BN))
             return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
         float* gb = epi.G + epi.off;
         const bool vec_ok = ((reinterpret_cast<uintptr_t>(gb) & 15u) == 0) && epi.ldrow % 4 == 0 && epi.ldG % 4 == 0;
+        // unaligned rows: the one-CTA-per-tile kernel (128-column tiles) with scalar stores
+        if (!vec_ok && !tc_make_map(&tb, B, rowsB, colsB, ldb, bk, 128))
+            return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
+        void* prof = profile_begin(PROF_DW, st, dw_bytes);
         if (!vec_ok) {
-            // unaligned rows: the one-CTA-per-tile kernel (128-column tiles) with scalar stores
-            if (!tc_make_map(&tb, B, rowsB, colsB, ldb, bk, 128))
-                return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
             e = bk == 64 ? launch_cfg<128, 64, 2, TC_DW, 4>(ta, tb, M, N, K, batch, kz, epi, status, st, 48 * 1024)
                          : launch_cfg<128, 32, 2, TC_DW, 4>(ta, tb, M, N, K, batch, kz, epi, status, st, 48 * 1024);
         } else {
             e = bk == 64 ? launch_dw<64, 2>(ta, tb, M, N, K, batch, status, gb, epi.ldrow, epi.ldG, st)
                          : launch_dw<32, 4>(ta, tb, M, N, K, batch, status, gb, epi.ldrow, epi.ldG, st);
         }
-        dw_profile_end(prof, st);
+        profile_end(prof, st);
     } else {
         if (!tc_make_map(&ta, A, rowsA, colsA, lda, 64, BM) || !tc_make_map(&tb, B, rowsB, colsB, ldb, 64, 256))
             return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
         // persistent: one CTA per SM (4 stages x 48 KB), 2 x 256 TMEM columns
+        void* prof = profile_begin(PROF_GEMM, st, 0.0);
         if (kind == TC_HIDDEN)
             e = launch_persistent<TC_HIDDEN>(ta, tb, M, N, K, epi, status, st);
         else if (kind == TC_LOGITS)
@@ -779,6 +780,7 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
             e = launch_persistent<TC_GBAR>(ta, tb, M, N, K, epi, status, st);
         else
             e = launch_persistent<TC_DX>(ta, tb, M, N, K, epi, status, st);
+        profile_end(prof, st);
     }
     if (e != cudaSuccess) return fail(DBW_ECUDA, "tc_gemm launch: %s", cudaGetErrorString(e));
     return DBW_OK;

@@ -90,6 +90,8 @@ _SIGS = {
     "dbw_choose_b": (_i32, [_vp, _f64, _f64, _i32, _vp, _vp, _vp]),
     "dbw_profile_dw": (_i32, [_i32]),
     "dbw_profile_dw_read": (_i32, [_vp, _vp, _vp]),
+    "dbw_profile_gemm": (_i32, [_i32]),
+    "dbw_profile_gemm_read": (_i32, [_vp, _vp]),
 }
 
 
@@ -321,6 +323,17 @@ def dbw_profile_dw_read():
     ms, n, b = C.c_double(), C.c_int64(), C.c_double()
     _check("dbw_profile_dw_read", lib().dbw_profile_dw_read(C.byref(ms), C.byref(n), C.byref(b)))
     return ms.value, n.value, b.value
+
+
+def dbw_profile_gemm(enable):
+    _check("dbw_profile_gemm", lib().dbw_profile_gemm(1 if enable else 0))
+
+
+def dbw_profile_gemm_read():
+    """(summed ms, launches) of the timed persistent tensor-core GEMM launches."""
+    ms, n = C.c_double(), C.c_int64()
+    _check("dbw_profile_gemm_read", lib().dbw_profile_gemm_read(C.byref(ms), C.byref(n)))
+    return ms.value, n.value
 
 
 # ----------------------------------------------------------------- helpers

@@ -268,3 +268,29 @@ def test_received_unsupported_shapes_are_refused():
             dbw.dbw_received_grads_update(wl.widths, prec, it.w, it.pool, it.labels, idx, n, B, mask, wl.lr, loss,
                                           part, it.ws)
         assert e.value.code == dbw.DBW_EUNSUPPORTED
+
+
+def test_launch_timing_channels():
+    """dbw_profile_gemm / dbw_profile_dw record one event pair per persistent GEMM and per
+    weight-gradient launch, only while enabled; a read forgets the records."""
+    L = len(RX_B32.widths) - 1
+    for received, gemms, dws in ((False, L + (L - 1), L), (True, L + L + (L - 1), 0)):
+        it = Iteration(RX_B32, static_b=2, received=received)
+        it.load_inputs(0)
+        it.step()
+        torch.cuda.synchronize()
+        dbw.dbw_profile_gemm(True)
+        dbw.dbw_profile_dw(True)
+        it.step()
+        torch.cuda.synchronize()
+        ms, launches = dbw.dbw_profile_gemm_read()
+        dms, dl, dbytes = dbw.dbw_profile_dw_read()
+        assert launches == gemms and ms > 0
+        assert dl == dws and (dws == 0 or (dms > 0 and dbytes > 0))
+        assert dbw.dbw_profile_gemm_read() == (0.0, 0)
+        dbw.dbw_profile_gemm(False)
+        dbw.dbw_profile_dw(False)
+        it.step()
+        torch.cuda.synchronize()
+        assert dbw.dbw_profile_gemm_read() == (0.0, 0)
+        assert dbw.dbw_profile_dw_read()[1] == 0
