@@ -444,6 +444,208 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
+// ------------------------------------------------------------------ CTA-pair persistent kernel
+// The persistent GEMM on CTA pairs: a cluster of two CTAs computes 256 x 256
+// output tiles with tcgen05.mma.cta_group::2.  CTA r of the pair stages rows
+// m0 + 128 r .. +127 of A and rows n0 + 128 r .. +127 of B (its half of the
+// tile's B) in its own shared memory; one thread of the even CTA issues the
+// MMAs, which read both CTAs' stages and accumulate output rows m0 + 128 r ..
+// into CTA r's TMEM.  Per SM a 64-deep stage is 32 KB for 128 x 256 x 64 MACs,
+// two thirds of what the single-CTA tile stages for the same work, so the ring
+// is deeper in the same shared memory and each SM pulls fewer bytes per flop.
+// Barriers (the same shared-memory offsets in both CTAs):
+//   full[s]    even CTA only: its producer arrives with the byte count of both
+//              CTAs' loads of stage s; the loads of both CTAs complete on it
+//   empty[s]   both CTAs: the MMA issuer's commit arrives on both
+//   tfull[a]   both CTAs: committed after the tile's last MMA into accumulator a
+//   tempty[a]  even CTA only: the four epilogue warps of each CTA arrive (8)
+// The epilogues are those of the single-CTA kernel, on 128-row sub-tiles.
+template <int KIND, int STAGES>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M,
+                        int N, int K, TcEpi epi, int* status) {
+    constexpr int BN = 256, BK = 64, SW = 128;
+    constexpr int A_BYTES = BM * BK * 2;          // 128 rows of A
+    constexpr int B_BYTES = (BN / 2) * BK * 2;    // this CTA's 128 rows of B
+    constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sA = smem;
+    uint8_t* sB = smem + STAGES * A_BYTES;
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+    uint64_t* empty_bar = full_bar + STAGES;
+    uint64_t* tfull_bar = empty_bar + STAGES;    // [2]
+    uint64_t* tempty_bar = tfull_bar + 2;        // [2]
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty_bar + 2);
+    int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_rank();
+    const long long pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+    int Meff = M, Keff = K, live_k = 1;
+    if (epi.kdev) {
+        live_k = *epi.kdev;
+        const long long r = static_cast<long long>(live_k > 0 ? live_k : 0) * epi.kmul;
+        if (KIND == TC_GBAR)
+            Keff = r < K ? static_cast<int>(r) : K;
+        else
+            Meff = r < M ? static_cast<int>(r) : M;
+    }
+    const int mt_n = (Meff + 2 * BM - 1) / (2 * BM), nt_n = (N + BN - 1) / BN;
+    const int msub_n = (M + BM - 1) / BM;   // 128-row sub-tiles of the full row extent
+    const long long total = live_k > 0 && Keff > 0 ? static_cast<long long>(mt_n) * nt_n : 0;
+    const int nk = (Keff + BK - 1) / BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(smem_u32(full_bar + s), 1);
+            mbar_init(smem_u32(empty_bar + s), 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(smem_u32(tfull_bar + a), 1);
+            mbar_init(smem_u32(tempty_bar + a), 8);
+        }
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tc2_alloc(smem_u32(tmem_slot), 2 * BN);
+        tc2_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();   // both CTAs' barriers exist before any remote arrive or load completes on them
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    volatile int* vabort = abort_flag;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer (both CTAs)
+        long long g = 0;
+        for (long long t = pair; t < total && !*vabort; t += npairs) {
+            const int ma = static_cast<int>(t / nt_n) * (2 * BM) + static_cast<int>(rank) * BM;
+            const int nb = static_cast<int>(t % nt_n) * BN + static_cast<int>(rank) * (BN / 2);
+            for (int kb = 0; kb < nk; ++kb, ++g) {
+                const int s = static_cast<int>(g % STAGES);
+                const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
+                if (!mbar_wait(smem_u32(empty_bar + s), ph ^ 1)) {
+                    atomicOr(status, 1);
+                    *vabort = 1;
+                    break;
+                }
+                if (rank == 0) mbar_expect_tx(smem_u32(full_bar + s), 2 * STAGE_BYTES);
+                const uint32_t bar = map_to_rank(smem_u32(full_bar + s), 0);
+                tma_load_2d_pair(smem_u32(sA + s * A_BYTES), &tmA, kb * BK, ma, bar);
+                tma_load_2d_pair(smem_u32(sB + s * B_BYTES), &tmB, kb * BK, nb, bar);
+            }
+        }
+        // the last use of every stage has been consumed: no load or commit is still
+        // on its way into this CTA's shared memory
+        if (!*vabort) {
+            for (long long q = g - STAGES < 0 ? 0 : g - STAGES; q < g; ++q) {
+                if (!mbar_wait(smem_u32(empty_bar + q % STAGES), static_cast<uint32_t>((q / STAGES) & 1))) {
+                    atomicOr(status, 1);
+                    *vabort = 1;
+                    break;
+                }
+            }
+        }
+    } else if (warp == 1 && lane == 0 && rank == 0) {
+        // ---------------- MMA issuer (even CTA)
+        constexpr uint32_t idesc = instr_desc_bf16(2 * BM, BN);
+        long long g = 0;
+        int i = 0;
+        for (long long t = pair; t < total && !*vabort; t += npairs, ++i) {
+            const int acc = i & 1;
+            const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
+            if (!mbar_wait(smem_u32(tempty_bar + acc), aph ^ 1)) {
+                atomicOr(status, 1);
+                *vabort = 1;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t dcol = tmem + static_cast<uint32_t>(acc * BN);
+            bool ok = true;
+            for (int kb = 0; kb < nk; ++kb, ++g) {
+                const int s = static_cast<int>(g % STAGES);
+                const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
+                if (!mbar_wait(smem_u32(full_bar + s), ph)) {
+                    atomicOr(status, 1);
+                    *vabort = 1;
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t a0 = smem_u32(sA + s * A_BYTES);
+                const uint32_t b0 = smem_u32(sB + s * B_BYTES);
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk)
+                    tc2_mma(dcol, smem_desc(a0 + kk * 32, SW), smem_desc(b0 + kk * 32, SW), idesc,
+                            (kb > 0 || kk > 0) ? 1u : 0u);
+                tc2_commit_multicast(smem_u32(empty_bar + s), 0x3);
+            }
+            tc2_commit_multicast(smem_u32(tfull_bar + acc), 0x3);
+            if (!ok) break;
+        }
+    } else if (warp >= 2) {
+        // ---------------- epilogue (both CTAs): 128-row sub-tile msub, TMEM lane quarter q
+        const int q = warp & 3;
+        int i = 0;
+        for (long long t = pair; t < total; t += npairs, ++i) {
+            const int acc = i & 1;
+            const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
+            if (!mbar_wait(smem_u32(tfull_bar + acc), aph)) {
+                atomicOr(status, 1);
+                *vabort = 1;
+                break;
+            }
+            if (*vabort) break;
+            tc_fence_after();
+            const int nt = static_cast<int>(t % nt_n);
+            const int msub = static_cast<int>(t / nt_n) * 2 + static_cast<int>(rank);
+            const int n0 = nt * BN;
+            const int row = msub * BM + q * 32 + lane;
+            const uint32_t tbase = tmem + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
+            double sq = 0.0;
+#pragma unroll 1
+            for (int c = 0; c < BN / 32; ++c) {
+                if (n0 + c * 32 >= N) break;
+                uint32_t r[32];
+                tc_ld_32cols(tbase + c * 32, r);
+                tc_wait_ld();
+                if constexpr (KIND == TC_GBAR)
+                    sq += gbar_chunk(epi, row, n0 + c * 32, M, N, 1.0f / static_cast<float>(live_k), r);
+                else
+                    epilogue_chunk<KIND>(epi, 0, row, n0 + c * 32, M, N, r);
+            }
+            if constexpr (KIND == TC_GBAR) {
+                // fixed-shape warp tree; one piece per (128-row sub-tile, column tile, quarter)
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+                if (lane == 0 && msub < msub_n) epi.pieces[(static_cast<long long>(msub) * nt_n + nt) * 4 + q] = sq;
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_remote(map_to_rank(smem_u32(tempty_bar + acc), 0));
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (*vabort && threadIdx.x == 0) {
+        // a wait ran out: give the pair's loads and MMAs still in flight time to land
+        // before the shared memory and the TMEM are released
+        const uint64_t t0 = globaltimer();
+        while (globaltimer() - t0 < 200000ull) {
+        }
+    }
+    __syncthreads();
+    cluster_sync();
+    if (warp == 0) {
+        tc_fence_after();
+        tc2_dealloc(tmem, 2 * BN);
+    }
+}
+
 // ------------------------------------------------------------------ persistent dW kernel
 // Per-worker weight gradient G[z*ldG + m*ldrow + n] = sum_{k < K} A[m, z*K + k] B[n, z*K + k]
 // (A = dZ^T [out, M], B = A_{l-1}^T [in, M], K = the worker's B samples).
@@ -667,6 +869,10 @@ cudaError_t launch_dw(const CUtensorMap& a, const CUtensorMap& b, int Mr, int Nr
     return cudaGetLastError();
 }
 
+#ifndef DBW_GEMM_CTA_PAIR
+#define DBW_GEMM_CTA_PAIR 1   // forward / input-gradient / mean-gradient GEMMs on CTA pairs
+#endif
+
 #ifndef DBW_PERSISTENT_STAGES
 #define DBW_PERSISTENT_STAGES 4   // TMA ring depth of the persistent GEMM (48 KB per stage)
 #endif
@@ -682,6 +888,50 @@ cudaError_t launch_persistent(const CUtensorMap& a, const CUtensorMap& b, int M,
     const long long tiles = static_cast<long long>((M + BM - 1) / BM) * ((N + 255) / 256);
     const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
     kern<<<grid, kThreads, Cfg::SMEM, st>>>(a, b, M, N, K, e, status);
+    return cudaGetLastError();
+}
+
+#ifndef DBW_PAIR_STAGES
+#define DBW_PAIR_STAGES 6   // TMA ring depth of the CTA-pair GEMM (32 KB per stage and CTA)
+#endif
+
+// Co-resident 2-CTA clusters of the pair kernel (the persistent grid), once per kind.
+template <class Kern>
+int pair_slots(Kern kern, int smem) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(2 * (sm_count() / 2), 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n < 1) {
+        cudaGetLastError();
+        n = sm_count() / 2;
+    }
+    return n;
+}
+
+template <int KIND>
+cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, const TcEpi& e, int* status,
+                        cudaStream_t st) {
+    constexpr int STAGES = DBW_PAIR_STAGES;
+    constexpr int SMEM = STAGES * (2 * BM * 64 * 2) + 256 + 1024;
+    static_assert(SMEM <= 227 * 1024, "pair ring does not fit in shared memory");
+    auto kern = tc_gemm_pair_kernel<KIND, STAGES>;
+    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
+    if (err != cudaSuccess) return err;
+    static int slots = 0;
+    static std::once_flag once;
+    std::call_once(once, [&] { slots = pair_slots(kern, SMEM); });
+    const long long tiles = static_cast<long long>((M + 2 * BM - 1) / (2 * BM)) * ((N + 255) / 256);
+    const int pairs = static_cast<int>(tiles < slots ? tiles : slots);
+    kern<<<2 * pairs, kThreads, SMEM, st>>>(a, b, M, N, K, e, status);
     return cudaGetLastError();
 }
 
@@ -768,6 +1018,20 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
         }
         profile_end(prof, st);
     } else {
+#if DBW_GEMM_CTA_PAIR
+        // CTA pairs: 256 x 256 tiles, each CTA stages 128 rows of A and 128 rows of B
+        if (!tc_make_map(&ta, A, rowsA, colsA, lda, 64, BM) || !tc_make_map(&tb, B, rowsB, colsB, ldb, 64, 128))
+            return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
+        void* prof = profile_begin(PROF_GEMM, st, 0.0);
+        if (kind == TC_HIDDEN)
+            e = launch_pair<TC_HIDDEN>(ta, tb, M, N, K, epi, status, st);
+        else if (kind == TC_LOGITS)
+            e = launch_pair<TC_LOGITS>(ta, tb, M, N, K, epi, status, st);
+        else if (kind == TC_GBAR)
+            e = launch_pair<TC_GBAR>(ta, tb, M, N, K, epi, status, st);
+        else
+            e = launch_pair<TC_DX>(ta, tb, M, N, K, epi, status, st);
+#else
         if (!tc_make_map(&ta, A, rowsA, colsA, lda, 64, BM) || !tc_make_map(&tb, B, rowsB, colsB, ldb, 64, 256))
             return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
         // persistent: one CTA per SM (4 stages x 48 KB), 2 x 256 TMEM columns
@@ -780,6 +1044,7 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
             e = launch_persistent<TC_GBAR>(ta, tb, M, N, K, epi, status, st);
         else
             e = launch_persistent<TC_DX>(ta, tb, M, N, K, epi, status, st);
+#endif
         profile_end(prof, st);
     }
     if (e != cudaSuccess) return fail(DBW_ECUDA, "tc_gemm launch: %s", cudaGetErrorString(e));
