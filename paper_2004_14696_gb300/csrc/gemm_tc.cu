@@ -34,61 +34,14 @@ constexpr int BM = 128;
 constexpr int kThreads = 192;
 
 // ------------------------------------------------------------------ epilogues
-// One thread: row ``row`` of the tile, 32 columns starting at ``nb``.
+// One thread: row ``row`` of the tile, 32 columns starting at ``nb`` (logits and the
+// one-CTA-per-tile weight-gradient kernel).
 template <int KIND>
 __device__ __forceinline__ void epilogue_chunk(const TcEpi& e, int z, int row, int nb, int M, int N,
                                                const uint32_t (&r)[32]) {
     if (row >= M) return;
     const bool full = nb + 32 <= N;
-    if (KIND == TC_HIDDEN || KIND == TC_DX) {
-        float x[32];
-        if (KIND == TC_HIDDEN) {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                const float v = u2f(r[j]) + (nb + j < N ? __ldg(e.bias + nb + j) : 0.f);
-                x[j] = v > 0.f ? v : 0.f;
-            }
-        } else {
-            const __nv_bfloat16* ap = e.act + static_cast<int64_t>(row) * e.ldact + nb;
-            if (full && ((reinterpret_cast<uintptr_t>(ap) & 15u) == 0)) {
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const uint4 raw = *reinterpret_cast<const uint4*>(ap + 8 * q);
-                    const __nv_bfloat16* h = reinterpret_cast<const __nv_bfloat16*>(&raw);
-#pragma unroll
-                    for (int t = 0; t < 8; ++t)
-                        x[8 * q + t] = u2f(r[8 * q + t]) * (__bfloat162float(h[t]) > 0.f ? 1.f : 0.f);
-                }
-            } else {
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    x[j] = (nb + j < N) ? u2f(r[j]) * (__bfloat162float(ap[j]) > 0.f ? 1.f : 0.f) : 0.f;
-            }
-        }
-        __nv_bfloat16* op = e.out + static_cast<int64_t>(row) * e.ldo + nb;
-        if (full && ((reinterpret_cast<uintptr_t>(op) & 15u) == 0)) {
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                uint4 w;
-                w.x = pack_bf16(x[8 * q + 0], x[8 * q + 1]);
-                w.y = pack_bf16(x[8 * q + 2], x[8 * q + 3]);
-                w.z = pack_bf16(x[8 * q + 4], x[8 * q + 5]);
-                w.w = pack_bf16(x[8 * q + 6], x[8 * q + 7]);
-                *reinterpret_cast<uint4*>(op + 8 * q) = w;
-            }
-        } else {
-#pragma unroll
-            for (int j = 0; j < 32; ++j)
-                if (nb + j < N) op[j] = __float2bfloat16_rn(x[j]);
-        }
-        if (e.outT) {
-            // column n of the tile -> row n of the transposed copy: the 32 lanes of the
-            // warp hold 32 consecutive rows m, so each store covers 64 contiguous bytes
-#pragma unroll
-            for (int j = 0; j < 32; ++j)
-                if (nb + j < N) e.outT[static_cast<int64_t>(nb + j) * e.ldT + row] = __float2bfloat16_rn(x[j]);
-        }
-    } else if (KIND == TC_LOGITS) {
+    if constexpr (KIND == TC_LOGITS) {
         float* op = e.outF + static_cast<int64_t>(row) * e.ldF + nb;
         if (full && ((reinterpret_cast<uintptr_t>(op) & 15u) == 0)) {
 #pragma unroll
@@ -106,6 +59,7 @@ __device__ __forceinline__ void epilogue_chunk(const TcEpi& e, int z, int row, i
                 if (nb + j < N) op[j] = u2f(r[j]) + __ldg(e.bias + nb + j);
         }
     } else {   // TC_DW: element (m, n) -> G[z*ldG + off + m*ldrow + n]
+        static_assert(KIND == TC_DW, "epilogue_chunk serves TC_LOGITS and TC_DW");
         float* op = e.G + static_cast<int64_t>(z) * e.ldG + e.off + static_cast<int64_t>(row) * e.ldrow + nb;
 #pragma unroll
         for (int j = 0; j < 32; ++j)
@@ -113,42 +67,160 @@ __device__ __forceinline__ void epilogue_chunk(const TcEpi& e, int z, int row, i
     }
 }
 
-// GBAR: one thread, row ``row`` (an output unit), 32 columns from ``nb``: the
-// mean over the k received workers, the SGD step and the chunk's sum of squares.
-__device__ __forceinline__ float gbar_chunk(const TcEpi& e, int row, int nb, int M, int N, float inv_k,
-                                            const uint32_t (&r)[32]) {
-    if (row >= M) return 0.f;
-    const int64_t at = e.off + static_cast<int64_t>(row) * e.ldrow + nb;
-    float* wp = e.W + at;
-    float* gp = e.gbar ? e.gbar + at : nullptr;
-    float sq = 0.f;
-    if (nb + 32 <= N && ((reinterpret_cast<uintptr_t>(wp) & 15u) == 0) &&
-        (!gp || ((reinterpret_cast<uintptr_t>(gp) & 15u) == 0))) {
+// ------------------------------------------------------------------ epilogues of the pair kernel
+// One thread owns one output row and 128 columns of a tile (four 32-column chunks
+// read from TMEM at ``taddr``).  The global loads a chunk needs (w for the SGD
+// step, the layer input for the ReLU mask) are issued one chunk ahead, so that
+// their latency overlaps the previous chunk's work.
+
+// bf16 activation chunk -> out (row-major) and, when asked, outT (transposed: the 32
+// lanes of a warp hold 32 consecutive rows, so each store covers 64 contiguous bytes).
+__device__ __forceinline__ void store_act_chunk(const TcEpi& e, int row, int nb, int N, const float (&x)[32]) {
+    __nv_bfloat16* op = e.out + static_cast<int64_t>(row) * e.ldo + nb;
+    if (nb + 32 <= N && ((reinterpret_cast<uintptr_t>(op) & 15u) == 0)) {
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            float4 g, wv = *reinterpret_cast<const float4*>(wp + 4 * q);
-            g.x = u2f(r[4 * q + 0]) * inv_k;
-            g.y = u2f(r[4 * q + 1]) * inv_k;
-            g.z = u2f(r[4 * q + 2]) * inv_k;
-            g.w = u2f(r[4 * q + 3]) * inv_k;
-            wv.x = fmaf(-e.lr, g.x, wv.x);
-            wv.y = fmaf(-e.lr, g.y, wv.y);
-            wv.z = fmaf(-e.lr, g.z, wv.z);
-            wv.w = fmaf(-e.lr, g.w, wv.w);
-            *reinterpret_cast<float4*>(wp + 4 * q) = wv;
-            if (gp) *reinterpret_cast<float4*>(gp + 4 * q) = g;
-            sq += g.x * g.x + g.y * g.y + g.z * g.z + g.w * g.w;
+        for (int q = 0; q < 4; ++q) {
+            uint4 w;
+            w.x = pack_bf16(x[8 * q + 0], x[8 * q + 1]);
+            w.y = pack_bf16(x[8 * q + 2], x[8 * q + 3]);
+            w.z = pack_bf16(x[8 * q + 4], x[8 * q + 5]);
+            w.w = pack_bf16(x[8 * q + 6], x[8 * q + 7]);
+            *reinterpret_cast<uint4*>(op + 8 * q) = w;
         }
     } else {
 #pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (nb + j < N) op[j] = __float2bfloat16_rn(x[j]);
+    }
+    if (e.outT) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (nb + j < N) e.outT[static_cast<int64_t>(nb + j) * e.ldT + row] = __float2bfloat16_rn(x[j]);
+    }
+}
+
+// TC_HIDDEN: A_l = ReLU(Z_l + b_l) in bf16.
+__device__ __forceinline__ void hidden_cols(const TcEpi& e, int row, int nb0, int M, int N, uint32_t taddr) {
+#pragma unroll 1
+    for (int c = 0; c < 4; ++c) {
+        const int nb = nb0 + 32 * c;
+        if (nb >= N) break;
+        uint32_t r[32];
+        tc_ld_32cols(taddr + 32 * c, r);
+        tc_wait_ld();
+        if (row >= M) continue;
+        float x[32];
+#pragma unroll
         for (int j = 0; j < 32; ++j) {
-            if (nb + j < N) {
-                const float g = u2f(r[j]) * inv_k;
-                wp[j] = fmaf(-e.lr, g, wp[j]);
-                if (gp) gp[j] = g;
-                sq += g * g;
+            const float v = u2f(r[j]) + (nb + j < N ? __ldg(e.bias + nb + j) : 0.f);
+            x[j] = v > 0.f ? v : 0.f;
+        }
+        store_act_chunk(e, row, nb, N, x);
+    }
+}
+
+// TC_DX: dZ_{l-1} = (dZ_l W_l) * 1[A_{l-1} > 0] in bf16; ``avec``: the act rows allow
+// 16-byte loads.
+__device__ __forceinline__ void dx_cols(const TcEpi& e, int row, int nb0, int M, int N, uint32_t taddr, bool avec) {
+    const bool rowok = row < M;
+    const __nv_bfloat16* ap = e.act + static_cast<int64_t>(row) * e.ldact + nb0;
+    uint4 nxt[4];
+    auto fetch = [&](int c) {
+        if (rowok && avec && nb0 + 32 * c + 32 <= N) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) nxt[j] = *reinterpret_cast<const uint4*>(ap + 32 * c + 8 * j);
+        }
+    };
+    fetch(0);
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+        const int nb = nb0 + 32 * c;
+        if (nb >= N) break;
+        uint4 cur[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) cur[j] = nxt[j];
+        if (c + 1 < 4) fetch(c + 1);
+        uint32_t r[32];
+        tc_ld_32cols(taddr + 32 * c, r);
+        tc_wait_ld();
+        if (!rowok) continue;
+        float x[32];
+        if (avec && nb + 32 <= N) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const __nv_bfloat16* hv = reinterpret_cast<const __nv_bfloat16*>(&cur[q]);
+#pragma unroll
+                for (int t = 0; t < 8; ++t)
+                    x[8 * q + t] = u2f(r[8 * q + t]) * (__bfloat162float(hv[t]) > 0.f ? 1.f : 0.f);
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                x[j] = (nb + j < N) ? u2f(r[j]) * (__bfloat162float(ap[32 * c + j]) > 0.f ? 1.f : 0.f) : 0.f;
+        }
+        store_act_chunk(e, row, nb, N, x);
+    }
+}
+
+// TC_GBAR: row ``row`` is an output unit; g = acc / k, w -= lr g, optional g out; returns
+// the sum of g^2 over the 128 columns (fp32 per chunk, fp64 across chunks).  ``wvec``:
+// w (and gbar) allow 16-byte accesses at every 32-column chunk.
+__device__ __forceinline__ double gbar_cols(const TcEpi& e, int row, int nb0, int M, int N, float inv_k,
+                                            uint32_t taddr, bool wvec) {
+    const bool rowok = row < M;
+    const int64_t at0 = e.off + static_cast<int64_t>(row) * e.ldrow + nb0;
+    float* wp = e.W + at0;
+    float* gp = e.gbar ? e.gbar + at0 : nullptr;
+    float4 nxt[8];
+    auto fetch = [&](int c) {
+        if (rowok && wvec && nb0 + 32 * c + 32 <= N) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) nxt[j] = *reinterpret_cast<const float4*>(wp + 32 * c + 4 * j);
+        }
+    };
+    fetch(0);
+    double sq = 0.0;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+        const int nb = nb0 + 32 * c;
+        if (nb >= N) break;
+        float4 cur[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) cur[j] = nxt[j];
+        if (c + 1 < 4) fetch(c + 1);
+        uint32_t r[32];
+        tc_ld_32cols(taddr + 32 * c, r);
+        tc_wait_ld();
+        if (!rowok) continue;
+        float part = 0.f;
+        if (wvec && nb + 32 <= N) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                float4 g, wv = cur[q];
+                g.x = u2f(r[4 * q + 0]) * inv_k;
+                g.y = u2f(r[4 * q + 1]) * inv_k;
+                g.z = u2f(r[4 * q + 2]) * inv_k;
+                g.w = u2f(r[4 * q + 3]) * inv_k;
+                wv.x = fmaf(-e.lr, g.x, wv.x);
+                wv.y = fmaf(-e.lr, g.y, wv.y);
+                wv.z = fmaf(-e.lr, g.z, wv.z);
+                wv.w = fmaf(-e.lr, g.w, wv.w);
+                *reinterpret_cast<float4*>(wp + 32 * c + 4 * q) = wv;
+                if (gp) *reinterpret_cast<float4*>(gp + 32 * c + 4 * q) = g;
+                part += g.x * g.x + g.y * g.y + g.z * g.z + g.w * g.w;
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                if (nb + j < N) {
+                    const float g = u2f(r[j]) * inv_k;
+                    wp[32 * c + j] = fmaf(-e.lr, g, wp[32 * c + j]);
+                    if (gp) gp[32 * c + j] = g;
+                    part += g * g;
+                }
             }
         }
+        sq += part;
     }
     return sq;
 }
@@ -275,175 +347,6 @@ __global__ void __launch_bounds__(kThreads, MINB)
     }
 }
 
-// ------------------------------------------------------------------ persistent GEMM kernel
-// The forward and input-gradient GEMMs (K = a layer width: long mainloops) as a
-// persistent kernel: one CTA per SM walks the 128 x 256 output tiles (n
-// fastest, so concurrently running CTAs share the A row block in L2), the TMA
-// ring of STAGES stages runs across tile boundaries, and two 256-column TMEM
-// accumulators let the fused epilogue of tile i (four warps, one per TMEM lane
-// quarter) overlap the mainloop of tile i+1.
-template <int KIND, int STAGES>
-__global__ void __launch_bounds__(kThreads, 1)
-    tc_gemm_persistent_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                              int M, int N, int K, TcEpi epi, int* status) {
-    using Cfg = TcCfg<256, 64, STAGES>;
-    constexpr int BN = 256, BK = 64;
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t* sA = smem;
-    uint8_t* sB = smem + STAGES * Cfg::A_BYTES;
-    uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
-    uint64_t* empty_bar = full_bar + STAGES;
-    uint64_t* tfull_bar = empty_bar + STAGES;    // [2]
-    uint64_t* tempty_bar = tfull_bar + 2;        // [2], 4 epilogue warps
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty_bar + 2);
-    int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
-
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // live extent: rows past (*kdev) * kmul of the row dimension are not computed
-    int Meff = M, Keff = K, live_k = 1;
-    if (epi.kdev) {
-        live_k = *epi.kdev;
-        const long long r = static_cast<long long>(live_k > 0 ? live_k : 0) * epi.kmul;
-        if (KIND == TC_GBAR)
-            Keff = r < K ? static_cast<int>(r) : K;
-        else
-            Meff = r < M ? static_cast<int>(r) : M;
-    }
-    const int mt_n = (Meff + BM - 1) / BM, nt_n = (N + BN - 1) / BN;
-    const long long total = live_k > 0 && Keff > 0 ? static_cast<long long>(mt_n) * nt_n : 0;
-    const int nk = (Keff + BK - 1) / BK;
-
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < STAGES; ++s) {
-            mbar_init(smem_u32(full_bar + s), 1);
-            mbar_init(smem_u32(empty_bar + s), 1);
-        }
-        for (int a = 0; a < 2; ++a) {
-            mbar_init(smem_u32(tfull_bar + a), 1);
-            mbar_init(smem_u32(tempty_bar + a), 4);
-        }
-        *abort_flag = 0;
-        fence_mbar_init();
-    }
-    if (warp == 0) {
-        tc_alloc(smem_u32(tmem_slot), 2 * BN);
-        tc_relinquish();
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = *tmem_slot;
-    volatile int* vabort = abort_flag;
-
-    if (warp == 0 && lane == 0) {
-        // ---------------- TMA producer
-        long long g = 0, issued = 0;
-        for (long long t = blockIdx.x; t < total && !*vabort; t += gridDim.x) {
-            const int m0 = static_cast<int>(t / nt_n) * BM, n0 = static_cast<int>(t % nt_n) * BN;
-            for (int kb = 0; kb < nk; ++kb, ++g) {
-                const int s = static_cast<int>(g % STAGES);
-                const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
-                if (!mbar_wait(smem_u32(empty_bar + s), ph ^ 1)) {
-                    atomicOr(status, 1);
-                    *vabort = 1;
-                    break;
-                }
-                mbar_expect_tx(smem_u32(full_bar + s), Cfg::STAGE_BYTES);
-                tma_load_2d(smem_u32(sA + s * Cfg::A_BYTES), &tmA, kb * BK, m0, smem_u32(full_bar + s));
-                tma_load_2d(smem_u32(sB + s * Cfg::B_BYTES), &tmB, kb * BK, n0, smem_u32(full_bar + s));
-                issued = g + 1;
-            }
-        }
-        if (*vabort) {
-            for (long long q = issued - STAGES < 0 ? 0 : issued - STAGES; q < issued; ++q)
-                mbar_wait(smem_u32(full_bar + q % STAGES), static_cast<uint32_t>((q / STAGES) & 1));
-        }
-    } else if (warp == 1 && lane == 0) {
-        // ---------------- MMA issuer
-        constexpr uint32_t idesc = instr_desc_bf16(BM, BN);
-        long long g = 0;
-        int i = 0;
-        for (long long t = blockIdx.x; t < total && !*vabort; t += gridDim.x, ++i) {
-            const int acc = i & 1;
-            const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
-            if (!mbar_wait(smem_u32(tempty_bar + acc), aph ^ 1)) {
-                atomicOr(status, 1);
-                *vabort = 1;
-                break;
-            }
-            tc_fence_after();
-            const uint32_t dcol = tmem + static_cast<uint32_t>(acc * BN);
-            bool ok = true;
-            for (int kb = 0; kb < nk; ++kb, ++g) {
-                const int s = static_cast<int>(g % STAGES);
-                const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
-                if (!mbar_wait(smem_u32(full_bar + s), ph)) {
-                    atomicOr(status, 1);
-                    *vabort = 1;
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t a0 = smem_u32(sA + s * Cfg::A_BYTES);
-                const uint32_t b0 = smem_u32(sB + s * Cfg::B_BYTES);
-#pragma unroll
-                for (int kk = 0; kk < BK / 16; ++kk)
-                    tc_mma(dcol, smem_desc(a0 + kk * 32, Cfg::SW), smem_desc(b0 + kk * 32, Cfg::SW), idesc,
-                           (kb > 0 || kk > 0) ? 1u : 0u);
-                tc_commit(smem_u32(empty_bar + s));
-            }
-            tc_commit(smem_u32(tfull_bar + acc));
-            if (!ok) break;
-        }
-    } else if (warp >= 2) {
-        // ---------------- epilogue
-        const int q = warp & 3;
-        int i = 0;
-        for (long long t = blockIdx.x; t < total; t += gridDim.x, ++i) {
-            const int acc = i & 1;
-            const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
-            if (!mbar_wait(smem_u32(tfull_bar + acc), aph)) {
-                atomicOr(status, 1);
-                *vabort = 1;
-                break;
-            }
-            if (*vabort) break;
-            tc_fence_after();
-            const int m0 = static_cast<int>(t / nt_n) * BM, n0 = static_cast<int>(t % nt_n) * BN;
-            const int row = m0 + q * 32 + lane;
-            const uint32_t tbase = tmem + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
-            double sq = 0.0;
-#pragma unroll 1
-            for (int c = 0; c < BN / 32; ++c) {
-                if (n0 + c * 32 >= N) break;
-                uint32_t r[32];
-                tc_ld_32cols(tbase + c * 32, r);
-                tc_wait_ld();
-                if constexpr (KIND == TC_GBAR)
-                    sq += gbar_chunk(epi, row, n0 + c * 32, M, N, 1.0f / static_cast<float>(live_k), r);
-                else
-                    epilogue_chunk<KIND>(epi, 0, row, n0 + c * 32, M, N, r);
-            }
-            if constexpr (KIND == TC_GBAR) {
-                // fixed-shape warp tree: the piece of (tile, quarter) does not depend on scheduling
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
-                if (lane == 0) epi.pieces[t * 4 + q] = sq;
-            }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(tempty_bar + acc));
-        }
-    }
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 0) {
-        tc_fence_after();
-        tc_dealloc(tmem, 2 * BN);
-    }
-}
-
 // ------------------------------------------------------------------ CTA-pair persistent kernel
 // The persistent GEMM on CTA pairs: a cluster of two CTAs computes 256 x 256
 // output tiles with tcgen05.mma.cta_group::2.  CTA r of the pair stages rows
@@ -458,10 +361,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 //              CTAs' loads of stage s; the loads of both CTAs complete on it
 //   empty[s]   both CTAs: the MMA issuer's commit arrives on both
 //   tfull[a]   both CTAs: committed after the tile's last MMA into accumulator a
-//   tempty[a]  even CTA only: the four epilogue warps of each CTA arrive (8)
-// The epilogues are those of the single-CTA kernel, on 128-row sub-tiles.
+//   tempty[a]  even CTA only: the eight epilogue warps of each CTA arrive (16)
+// Ten warps: 0 TMA producer and TMEM owner, 1 MMA issuer (even CTA), 2-9 epilogue:
+// warp w reads TMEM lane quarter w % 4 (32 rows of the CTA's 128-row sub-tile) and
+// the columns [128 h, 128 h + 128) of the tile, h = (w - 2) / 4.
+constexpr int kPairThreads = 320;
+
 template <int KIND, int STAGES>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M,
                         int N, int K, TcEpi epi, int* status) {
     constexpr int BN = 256, BK = 64, SW = 128;
@@ -503,7 +410,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(smem_u32(tfull_bar + a), 1);
-            mbar_init(smem_u32(tempty_bar + a), 8);
+            mbar_init(smem_u32(tempty_bar + a), 16);
         }
         *abort_flag = 0;
         fence_mbar_init();
@@ -588,8 +495,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             if (!ok) break;
         }
     } else if (warp >= 2) {
-        // ---------------- epilogue (both CTAs): 128-row sub-tile msub, TMEM lane quarter q
-        const int q = warp & 3;
+        // ---------------- epilogue (both CTAs): 128-row sub-tile msub, lane quarter q, column half h
+        const int q = warp & 3, h = (warp - 2) >> 2;
+        const bool wvec = KIND == TC_GBAR && ((reinterpret_cast<uintptr_t>(epi.W) & 15u) == 0) &&
+                          ((reinterpret_cast<uintptr_t>(epi.gbar) & 15u) == 0) && epi.off % 4 == 0 &&
+                          epi.ldrow % 4 == 0;
+        const bool avec = KIND == TC_DX && ((reinterpret_cast<uintptr_t>(epi.act) & 15u) == 0) && epi.ldact % 8 == 0;
+        const float inv_k = 1.0f / static_cast<float>(live_k);
         int i = 0;
         for (long long t = pair; t < total; t += npairs, ++i) {
             const int acc = i & 1;
@@ -603,26 +515,30 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const int nt = static_cast<int>(t % nt_n);
             const int msub = static_cast<int>(t / nt_n) * 2 + static_cast<int>(rank);
-            const int n0 = nt * BN;
+            const int nb0 = nt * BN + h * (BN / 2);
             const int row = msub * BM + q * 32 + lane;
-            const uint32_t tbase = tmem + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
-            double sq = 0.0;
-#pragma unroll 1
-            for (int c = 0; c < BN / 32; ++c) {
-                if (n0 + c * 32 >= N) break;
-                uint32_t r[32];
-                tc_ld_32cols(tbase + c * 32, r);
-                tc_wait_ld();
-                if constexpr (KIND == TC_GBAR)
-                    sq += gbar_chunk(epi, row, n0 + c * 32, M, N, 1.0f / static_cast<float>(live_k), r);
-                else
-                    epilogue_chunk<KIND>(epi, 0, row, n0 + c * 32, M, N, r);
-            }
+            const uint32_t taddr = tmem + static_cast<uint32_t>(acc * BN + h * (BN / 2)) +
+                                   (static_cast<uint32_t>(q * 32) << 16);
             if constexpr (KIND == TC_GBAR) {
-                // fixed-shape warp tree; one piece per (128-row sub-tile, column tile, quarter)
+                double sq = gbar_cols(epi, row, nb0, M, N, inv_k, taddr, wvec);
+                // fixed-shape warp tree; one piece per (128-row sub-tile, column tile, half, quarter)
 #pragma unroll
                 for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
-                if (lane == 0 && msub < msub_n) epi.pieces[(static_cast<long long>(msub) * nt_n + nt) * 4 + q] = sq;
+                if (lane == 0 && msub < msub_n)
+                    epi.pieces[(static_cast<long long>(msub) * nt_n + nt) * 8 + h * 4 + q] = sq;
+            } else if constexpr (KIND == TC_DX) {
+                dx_cols(epi, row, nb0, M, N, taddr, avec);
+            } else if constexpr (KIND == TC_HIDDEN) {
+                hidden_cols(epi, row, nb0, M, N, taddr);
+            } else {
+#pragma unroll 1
+                for (int c = 0; c < 4; ++c) {
+                    if (nb0 + c * 32 >= N) break;
+                    uint32_t r[32];
+                    tc_ld_32cols(taddr + c * 32, r);
+                    tc_wait_ld();
+                    epilogue_chunk<KIND>(epi, 0, row, nb0 + c * 32, M, N, r);
+                }
             }
             tc_fence_before();
             __syncwarp();
@@ -869,28 +785,6 @@ cudaError_t launch_dw(const CUtensorMap& a, const CUtensorMap& b, int Mr, int Nr
     return cudaGetLastError();
 }
 
-#ifndef DBW_GEMM_CTA_PAIR
-#define DBW_GEMM_CTA_PAIR 1   // forward / input-gradient / mean-gradient GEMMs on CTA pairs
-#endif
-
-#ifndef DBW_PERSISTENT_STAGES
-#define DBW_PERSISTENT_STAGES 4   // TMA ring depth of the persistent GEMM (48 KB per stage)
-#endif
-
-template <int KIND>
-cudaError_t launch_persistent(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, const TcEpi& e,
-                              int* status, cudaStream_t st) {
-    constexpr int STAGES = DBW_PERSISTENT_STAGES;
-    using Cfg = TcCfg<256, 64, STAGES>;
-    auto kern = tc_gemm_persistent_kernel<KIND, STAGES>;
-    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::SMEM);
-    if (err != cudaSuccess) return err;
-    const long long tiles = static_cast<long long>((M + BM - 1) / BM) * ((N + 255) / 256);
-    const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
-    kern<<<grid, kThreads, Cfg::SMEM, st>>>(a, b, M, N, K, e, status);
-    return cudaGetLastError();
-}
-
 #ifndef DBW_PAIR_STAGES
 #define DBW_PAIR_STAGES 6   // TMA ring depth of the CTA-pair GEMM (32 KB per stage and CTA)
 #endif
@@ -905,7 +799,7 @@ int pair_slots(Kern kern, int smem) {
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     cfg.gridDim = dim3(2 * (sm_count() / 2), 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.blockDim = dim3(kPairThreads, 1, 1);
     cfg.dynamicSmemBytes = smem;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
@@ -931,7 +825,7 @@ cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, int M, int N
     std::call_once(once, [&] { slots = pair_slots(kern, SMEM); });
     const long long tiles = static_cast<long long>((M + 2 * BM - 1) / (2 * BM)) * ((N + 255) / 256);
     const int pairs = static_cast<int>(tiles < slots ? tiles : slots);
-    kern<<<2 * pairs, kThreads, SMEM, st>>>(a, b, M, N, K, e, status);
+    kern<<<2 * pairs, kPairThreads, SMEM, st>>>(a, b, M, N, K, e, status);
     return cudaGetLastError();
 }
 
@@ -1018,7 +912,6 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
         }
         profile_end(prof, st);
     } else {
-#if DBW_GEMM_CTA_PAIR
         // CTA pairs: 256 x 256 tiles, each CTA stages 128 rows of A and 128 rows of B
         if (!tc_make_map(&ta, A, rowsA, colsA, lda, 64, BM) || !tc_make_map(&tb, B, rowsB, colsB, ldb, 64, 128))
             return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
@@ -1031,20 +924,6 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
             e = launch_pair<TC_GBAR>(ta, tb, M, N, K, epi, status, st);
         else
             e = launch_pair<TC_DX>(ta, tb, M, N, K, epi, status, st);
-#else
-        if (!tc_make_map(&ta, A, rowsA, colsA, lda, 64, BM) || !tc_make_map(&tb, B, rowsB, colsB, ldb, 64, 256))
-            return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
-        // persistent: one CTA per SM (4 stages x 48 KB), 2 x 256 TMEM columns
-        void* prof = profile_begin(PROF_GEMM, st, 0.0);
-        if (kind == TC_HIDDEN)
-            e = launch_persistent<TC_HIDDEN>(ta, tb, M, N, K, epi, status, st);
-        else if (kind == TC_LOGITS)
-            e = launch_persistent<TC_LOGITS>(ta, tb, M, N, K, epi, status, st);
-        else if (kind == TC_GBAR)
-            e = launch_persistent<TC_GBAR>(ta, tb, M, N, K, epi, status, st);
-        else
-            e = launch_persistent<TC_DX>(ta, tb, M, N, K, epi, status, st);
-#endif
         profile_end(prof, st);
     }
     if (e != cudaSuccess) return fail(DBW_ECUDA, "tc_gemm launch: %s", cudaGetErrorString(e));

@@ -27,7 +27,8 @@ struct TcEpi {
     int64_t ldG, off, ldrow;
     // GBAR (mean over the received workers, Eqs. (3)-(4)): with g = acc / k,
     // W[off + m * ldrow + n] -= lr * g, gbar[off + m * ldrow + n] = g (nullable), and the
-    // tile's sum of g^2 (fp64) into pieces[tile * 4 + q] for TMEM lane quarter q.
+    // sums of g^2 (fp64) into pieces[(s * ceil(N / 256) + nt) * 8 + h * 4 + q]: rows
+    // 128 s + 32 q .. +31 (s < ceil(M / 128)), columns 256 nt + 128 h .. +127.
     float* W;
     float* gbar;
     float lr;
@@ -66,8 +67,13 @@ bool tc_shape_ok(int64_t lda, int64_t ldb, int K, int64_t kz, const void* A, con
 //   (D D^T)[r, c] * ((A A^T)[r, c] + 1)
 // for the row groups of the first (*kdev) * B rows.  A = act [rows, ldA] (K = colsA),
 // D = dz [rows, ldD] (K = colsD), both bf16 row-major; B % 32 == 0 and either
-// 128 % B == 0 or B % 128 == 0.
+// 128 % B == 0 or B % 128 == 0.  part: tc_gram_partial_floats(rows, B) floats of
+// scratch for the partial products of the K ranges; cnt: tc_gram_items(rows, B)
+// int32 counters, zero on entry and left zero on return.
 int tc_gram(const __nv_bfloat16* act, int64_t ldA, int64_t colsA, const __nv_bfloat16* dz, int64_t ldD,
-            int64_t colsD, int rows, int B, const int* kdev, double* pieces, int* status, cudaStream_t st);
+            int64_t colsD, int rows, int B, const int* kdev, double* pieces, float* part, int* cnt, int* status,
+            cudaStream_t st);
+size_t tc_gram_partial_floats(int rows, int B);
+size_t tc_gram_items(int rows, int B);
 
 }  // namespace dbw

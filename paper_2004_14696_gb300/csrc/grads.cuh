@@ -60,11 +60,14 @@ struct RxPlan {
     size_t off_sel;                    // int32 [n]: received workers, increasing
     size_t off_k;                      // int32: k
     size_t off_bpart;                  // fp32 [ceil(M / 256), max out]: bias column sums per 256-row chunk
-    size_t off_pw[DBW_LMAX];           // fp64 [tiles_l * 4]: pieces of ||g_t(W_l)||^2
+    size_t off_pw[DBW_LMAX];           // fp64 [tiles_l * 8]: pieces of ||g_t(W_l)||^2
     int64_t npw[DBW_LMAX];
     size_t off_pb[DBW_LMAX];           // fp64 [ceil(out_l / 256)]: pieces of ||g_t(b_l)||^2
     int npb[DBW_LMAX];
     size_t off_pg[DBW_LMAX];           // fp64 [(M / 32) * CT]: Gram pieces of ||g_j||^2
+    size_t off_gpart;                  // fp32: partial Gram products of the K ranges (shared by the layers)
+    size_t off_gcnt;                   // int32 [gram items]: per-item range counters, zeroed at the start of a call
+    int ngcnt;
     size_t ws_bytes;
 };
 

@@ -244,9 +244,11 @@ __global__ void bias_grad_ld_kernel(const __nv_bfloat16* __restrict__ dZ, int64_
 // 1024 threads: a ballot prefix count per warp, then over the warp totals.
 __global__ void __launch_bounds__(1024) compact_received_kernel(const uint8_t* __restrict__ mask, int n,
                                                                 int32_t* __restrict__ sel, int* __restrict__ kout,
-                                                                float* __restrict__ loss) {
+                                                                float* __restrict__ loss, int* __restrict__ zero,
+                                                                int nzero) {
     __shared__ int warp_tot[32];
     const int j = threadIdx.x, lane = j & 31, warp = j >> 5;
+    for (int q = j; q < nzero; q += blockDim.x) zero[q] = 0;
     const bool on = j < n && mask[j] != 0;
     const unsigned bal = __ballot_sync(0xffffffffu, on);
     if (lane == 0) warp_tot[warp] = __popc(bal);
@@ -562,12 +564,15 @@ bool make_rx_plan(int L, const int32_t* widths, int n, int B, RxPlan* P) {
     P->off_bpart = take(static_cast<size_t>((g.M + 255) / 256) * maxout * 4);
     for (int l = 0; l < L; ++l) {
         const int fin = g.widths[l], fout = g.widths[l + 1];
-        P->npw[l] = static_cast<int64_t>((fout + 127) / 128) * ((fin + 255) / 256) * 4;
+        P->npw[l] = static_cast<int64_t>((fout + 127) / 128) * ((fin + 255) / 256) * 8;
         P->off_pw[l] = take(static_cast<size_t>(P->npw[l]) * 8);
         P->npb[l] = (fout + 255) / 256;
         P->off_pb[l] = take(static_cast<size_t>(P->npb[l]) * 8);
         P->off_pg[l] = take(static_cast<size_t>(g.M / 32) * P->CT * 8);
     }
+    P->off_gpart = take(tc_gram_partial_floats(g.M, B) * 4);
+    P->ngcnt = static_cast<int>(tc_gram_items(g.M, B));
+    P->off_gcnt = take(static_cast<size_t>(P->ngcnt) * 4);
     P->ws_bytes = cur;
     return true;
 }
@@ -588,7 +593,9 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
     cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int), st);
     if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
 
-    compact_received_kernel<<<1, 1024, 0, st>>>(mask, n, sel, kdev, loss);
+    int* gcnt = reinterpret_cast<int*>(ws + P.off_gcnt);
+    float* gpart = reinterpret_cast<float*>(ws + P.off_gpart);
+    compact_received_kernel<<<1, 1024, 0, st>>>(mask, n, sel, kdev, loss, gcnt, P.ngcnt);
     for (int l = 0; l < L; ++l) {
         const int fin = g.widths[l], fout = g.widths[l + 1];
         dim3 grid((fin + 63) / 64, (fout + 63) / 64);
@@ -663,7 +670,7 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
         e = cudaGetLastError();
         if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
         rc = tc_gram(bf(T.off_act[l]), T.ldact[l], fin, bf(T.off_dz[cur]), T.ldz, fout, M, B, kdev, f64(P.off_pg[l]),
-                     status, st);
+                     gpart, gcnt, status, st);
         if (rc) return rc;
         if (l > 0) {
             TcEpi ex{};
