@@ -42,27 +42,36 @@ __global__ void __launch_bounds__(256) cast_transpose_tile_kernel(const float* _
     const int live = rowmap.live(rows);
     if (m0 >= live) return;
     const int t = threadIdx.x;
+    // all four rows' loads first, so that each thread has 64 bytes in flight
+    float v[4][4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
         const int e = t + 256 * q;
         const int r = e >> 4, c = c0 + 4 * (e & 15);
         const int m = m0 + r;
-        float v[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) v[q][j] = 0.f;
         if (m < live && c < cols) {
             const int64_t sr = rowmap(m);
             if (sr >= 0) {
                 const float* p = src + sr * lds + c;
                 if (c + 3 < cols && ((reinterpret_cast<uintptr_t>(p) & 15u) == 0)) {
-                    const float4 f = *reinterpret_cast<const float4*>(p);
-                    v[0] = f.x, v[1] = f.y, v[2] = f.z, v[3] = f.w;
+                    const float4 f = __ldcs(reinterpret_cast<const float4*>(p));
+                    v[q][0] = f.x, v[q][1] = f.y, v[q][2] = f.z, v[q][3] = f.w;
                 } else {
-                    for (int j = 0; j < 4 && c + j < cols; ++j) v[j] = p[j];
+                    for (int j = 0; j < 4 && c + j < cols; ++j) v[q][j] = p[j];
                 }
             }
         }
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int e = t + 256 * q;
+        const int r = e >> 4, c = c0 + 4 * (e & 15);
+        const int m = m0 + r;
         __nv_bfloat16 h[4];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) h[j] = __float2bfloat16_rn(v[j]);
+        for (int j = 0; j < 4; ++j) h[j] = __float2bfloat16_rn(v[q][j]);
 #pragma unroll
         for (int j = 0; j < 4; ++j) tile[r][4 * (e & 15) + j] = h[j];
         if (m < live && c < cols) {
