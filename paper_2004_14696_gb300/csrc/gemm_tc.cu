@@ -356,6 +356,11 @@ __global__ void __launch_bounds__(kThreads, MINB)
 // into CTA r's TMEM.  Per SM a 64-deep stage is 32 KB for 128 x 256 x 64 MACs,
 // two thirds of what the single-CTA tile stages for the same work, so the ring
 // is deeper in the same shared memory and each SM pulls fewer bytes per flop.
+//
+// One launch may carry two independent problems (KIND1 != KIND0 or p[1] live):
+// their tiles form one list, those of problem 0 first, dealt to the pairs in
+// turn, so that the second problem fills the last partial wave of the first.
+//
 // Barriers (the same shared-memory offsets in both CTAs):
 //   full[s]    even CTA only: its producer arrives with the byte count of both
 //              CTAs' loads of stage s; the loads of both CTAs complete on it
@@ -367,10 +372,85 @@ __global__ void __launch_bounds__(kThreads, MINB)
 // the columns [128 h, 128 h + 128) of the tile, h = (w - 2) / 4.
 constexpr int kPairThreads = 320;
 
-template <int KIND, int STAGES>
+struct PairProblem {
+    CUtensorMap tmA, tmB;
+    int M, N, K;
+    TcEpi epi;
+};
+struct PairArgs {
+    PairProblem p[2];
+    int nprob;        // 1 or 2
+    int* status;
+};
+
+// Live extent of one problem: rows past (*kdev) * kmul of the row dimension (M, or
+// K for GBAR) are not computed.
+struct PairShape {
+    int Meff, Keff, live_k, mt_n, nt_n, msub_n, nk;
+    long long tiles;
+};
+template <int KIND>
+__device__ __forceinline__ PairShape pair_shape(const PairProblem& P) {
+    constexpr int BN = 256, BK = 64;
+    PairShape S;
+    S.Meff = P.M;
+    S.Keff = P.K;
+    S.live_k = 1;
+    if (P.epi.kdev) {
+        S.live_k = *P.epi.kdev;
+        const long long r = static_cast<long long>(S.live_k > 0 ? S.live_k : 0) * P.epi.kmul;
+        if (KIND == TC_GBAR)
+            S.Keff = r < P.K ? static_cast<int>(r) : P.K;
+        else
+            S.Meff = r < P.M ? static_cast<int>(r) : P.M;
+    }
+    S.mt_n = (S.Meff + 2 * BM - 1) / (2 * BM);
+    S.nt_n = (P.N + BN - 1) / BN;
+    S.msub_n = (P.M + BM - 1) / BM;   // 128-row sub-tiles of the full row extent
+    S.tiles = S.live_k > 0 && S.Keff > 0 ? static_cast<long long>(S.mt_n) * S.nt_n : 0;
+    S.nk = (S.Keff + BK - 1) / BK;
+    return S;
+}
+
+// Epilogue of one tile for problem kind KIND (one thread: one row, 128 columns).
+template <int KIND>
+__device__ __forceinline__ void pair_epilogue(const PairProblem& P, const PairShape& S, long long t, int rank, int q,
+                                              int h, int lane, uint32_t taddr) {
+    constexpr int BN = 256;
+    const TcEpi& epi = P.epi;
+    const int nt = static_cast<int>(t % S.nt_n);
+    const int msub = static_cast<int>(t / S.nt_n) * 2 + rank;
+    const int nb0 = nt * BN + h * (BN / 2);
+    const int row = msub * BM + q * 32 + lane;
+    if constexpr (KIND == TC_GBAR) {
+        const bool wvec = ((reinterpret_cast<uintptr_t>(epi.W) & 15u) == 0) &&
+                          ((reinterpret_cast<uintptr_t>(epi.gbar) & 15u) == 0) && epi.off % 4 == 0 &&
+                          epi.ldrow % 4 == 0;
+        double sq = gbar_cols(epi, row, nb0, P.M, P.N, 1.0f / static_cast<float>(S.live_k), taddr, wvec);
+        // fixed-shape warp tree; one piece per (128-row sub-tile, column tile, half, quarter)
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+        if (lane == 0 && msub < S.msub_n) epi.pieces[(static_cast<long long>(msub) * S.nt_n + nt) * 8 + h * 4 + q] = sq;
+    } else if constexpr (KIND == TC_DX) {
+        const bool avec = ((reinterpret_cast<uintptr_t>(epi.act) & 15u) == 0) && epi.ldact % 8 == 0;
+        dx_cols(epi, row, nb0, P.M, P.N, taddr, avec);
+    } else if constexpr (KIND == TC_HIDDEN) {
+        hidden_cols(epi, row, nb0, P.M, P.N, taddr);
+    } else {
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+            if (nb0 + c * 32 >= P.N) break;
+            uint32_t r[32];
+            tc_ld_32cols(taddr + c * 32, r);
+            tc_wait_ld();
+            epilogue_chunk<KIND>(epi, 0, row, nb0 + c * 32, P.M, P.N, r);
+        }
+    }
+}
+
+template <int KIND0, int KIND1, int STAGES>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
-    tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M,
-                        int N, int K, TcEpi epi, int* status) {
+    tc_gemm_pair_kernel(const __grid_constant__ PairArgs args) {
     constexpr int BN = 256, BK = 64, SW = 128;
     constexpr int A_BYTES = BM * BK * 2;          // 128 rows of A
     constexpr int B_BYTES = (BN / 2) * BK * 2;    // this CTA's 128 rows of B
@@ -389,19 +469,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t rank = cluster_rank();
     const long long pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
-    int Meff = M, Keff = K, live_k = 1;
-    if (epi.kdev) {
-        live_k = *epi.kdev;
-        const long long r = static_cast<long long>(live_k > 0 ? live_k : 0) * epi.kmul;
-        if (KIND == TC_GBAR)
-            Keff = r < K ? static_cast<int>(r) : K;
-        else
-            Meff = r < M ? static_cast<int>(r) : M;
-    }
-    const int mt_n = (Meff + 2 * BM - 1) / (2 * BM), nt_n = (N + BN - 1) / BN;
-    const int msub_n = (M + BM - 1) / BM;   // 128-row sub-tiles of the full row extent
-    const long long total = live_k > 0 && Keff > 0 ? static_cast<long long>(mt_n) * nt_n : 0;
-    const int nk = (Keff + BK - 1) / BK;
+    int* status = args.status;
+    const PairShape S0 = pair_shape<KIND0>(args.p[0]);
+    PairShape S1 = S0;
+    S1.tiles = 0;
+    if (args.nprob > 1) S1 = pair_shape<KIND1>(args.p[1]);
+    const long long total = S0.tiles + S1.tiles;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -430,9 +503,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         // ---------------- TMA producer (both CTAs)
         long long g = 0;
         for (long long t = pair; t < total && !*vabort; t += npairs) {
-            const int ma = static_cast<int>(t / nt_n) * (2 * BM) + static_cast<int>(rank) * BM;
-            const int nb = static_cast<int>(t % nt_n) * BN + static_cast<int>(rank) * (BN / 2);
-            for (int kb = 0; kb < nk; ++kb, ++g) {
+            const bool second = t >= S0.tiles;
+            const long long u = second ? t - S0.tiles : t;
+            const PairShape& S = second ? S1 : S0;
+            const CUtensorMap* tmA = second ? &args.p[1].tmA : &args.p[0].tmA;
+            const CUtensorMap* tmB = second ? &args.p[1].tmB : &args.p[0].tmB;
+            const int ma = static_cast<int>(u / S.nt_n) * (2 * BM) + static_cast<int>(rank) * BM;
+            const int nb = static_cast<int>(u % S.nt_n) * BN + static_cast<int>(rank) * (BN / 2);
+            for (int kb = 0; kb < S.nk; ++kb, ++g) {
                 const int s = static_cast<int>(g % STAGES);
                 const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
                 if (!mbar_wait(smem_u32(empty_bar + s), ph ^ 1)) {
@@ -442,8 +520,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
                 }
                 if (rank == 0) mbar_expect_tx(smem_u32(full_bar + s), 2 * STAGE_BYTES);
                 const uint32_t bar = map_to_rank(smem_u32(full_bar + s), 0);
-                tma_load_2d_pair(smem_u32(sA + s * A_BYTES), &tmA, kb * BK, ma, bar);
-                tma_load_2d_pair(smem_u32(sB + s * B_BYTES), &tmB, kb * BK, nb, bar);
+                tma_load_2d_pair(smem_u32(sA + s * A_BYTES), tmA, kb * BK, ma, bar);
+                tma_load_2d_pair(smem_u32(sB + s * B_BYTES), tmB, kb * BK, nb, bar);
             }
         }
         // the last use of every stage has been consumed: no load or commit is still
@@ -463,6 +541,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         long long g = 0;
         int i = 0;
         for (long long t = pair; t < total && !*vabort; t += npairs, ++i) {
+            const int nk = t >= S0.tiles ? S1.nk : S0.nk;
             const int acc = i & 1;
             const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
             if (!mbar_wait(smem_u32(tempty_bar + acc), aph ^ 1)) {
@@ -497,11 +576,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     } else if (warp >= 2) {
         // ---------------- epilogue (both CTAs): 128-row sub-tile msub, lane quarter q, column half h
         const int q = warp & 3, h = (warp - 2) >> 2;
-        const bool wvec = KIND == TC_GBAR && ((reinterpret_cast<uintptr_t>(epi.W) & 15u) == 0) &&
-                          ((reinterpret_cast<uintptr_t>(epi.gbar) & 15u) == 0) && epi.off % 4 == 0 &&
-                          epi.ldrow % 4 == 0;
-        const bool avec = KIND == TC_DX && ((reinterpret_cast<uintptr_t>(epi.act) & 15u) == 0) && epi.ldact % 8 == 0;
-        const float inv_k = 1.0f / static_cast<float>(live_k);
         int i = 0;
         for (long long t = pair; t < total; t += npairs, ++i) {
             const int acc = i & 1;
@@ -513,33 +587,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
             }
             if (*vabort) break;
             tc_fence_after();
-            const int nt = static_cast<int>(t % nt_n);
-            const int msub = static_cast<int>(t / nt_n) * 2 + static_cast<int>(rank);
-            const int nb0 = nt * BN + h * (BN / 2);
-            const int row = msub * BM + q * 32 + lane;
             const uint32_t taddr = tmem + static_cast<uint32_t>(acc * BN + h * (BN / 2)) +
                                    (static_cast<uint32_t>(q * 32) << 16);
-            if constexpr (KIND == TC_GBAR) {
-                double sq = gbar_cols(epi, row, nb0, M, N, inv_k, taddr, wvec);
-                // fixed-shape warp tree; one piece per (128-row sub-tile, column tile, half, quarter)
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
-                if (lane == 0 && msub < msub_n)
-                    epi.pieces[(static_cast<long long>(msub) * nt_n + nt) * 8 + h * 4 + q] = sq;
-            } else if constexpr (KIND == TC_DX) {
-                dx_cols(epi, row, nb0, M, N, taddr, avec);
-            } else if constexpr (KIND == TC_HIDDEN) {
-                hidden_cols(epi, row, nb0, M, N, taddr);
-            } else {
-#pragma unroll 1
-                for (int c = 0; c < 4; ++c) {
-                    if (nb0 + c * 32 >= N) break;
-                    uint32_t r[32];
-                    tc_ld_32cols(taddr + c * 32, r);
-                    tc_wait_ld();
-                    epilogue_chunk<KIND>(epi, 0, row, nb0 + c * 32, M, N, r);
-                }
-            }
+            if (t < S0.tiles)
+                pair_epilogue<KIND0>(args.p[0], S0, t, static_cast<int>(rank), q, h, lane, taddr);
+            else
+                pair_epilogue<KIND1>(args.p[1], S1, t - S0.tiles, static_cast<int>(rank), q, h, lane, taddr);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_remote(map_to_rank(smem_u32(tempty_bar + acc), 0));
@@ -811,21 +864,23 @@ int pair_slots(Kern kern, int smem) {
     return n;
 }
 
-template <int KIND>
-cudaError_t launch_pair(const CUtensorMap& a, const CUtensorMap& b, int M, int N, int K, const TcEpi& e, int* status,
-                        cudaStream_t st) {
+template <int KIND0, int KIND1>
+cudaError_t launch_pair(const PairArgs& args, cudaStream_t st) {
     constexpr int STAGES = DBW_PAIR_STAGES;
     constexpr int SMEM = STAGES * (2 * BM * 64 * 2) + 256 + 1024;
     static_assert(SMEM <= 227 * 1024, "pair ring does not fit in shared memory");
-    auto kern = tc_gemm_pair_kernel<KIND, STAGES>;
+    auto kern = tc_gemm_pair_kernel<KIND0, KIND1, STAGES>;
     cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
     if (err != cudaSuccess) return err;
     static int slots = 0;
     static std::once_flag once;
     std::call_once(once, [&] { slots = pair_slots(kern, SMEM); });
-    const long long tiles = static_cast<long long>((M + 2 * BM - 1) / (2 * BM)) * ((N + 255) / 256);
+    long long tiles = 0;   // upper bound: the live extents are read on the device
+    for (int i = 0; i < args.nprob; ++i)
+        tiles += static_cast<long long>((args.p[i].M + 2 * BM - 1) / (2 * BM)) * ((args.p[i].N + 255) / 256);
     const int pairs = static_cast<int>(tiles < slots ? tiles : slots);
-    kern<<<2 * pairs, kPairThreads, SMEM, st>>>(a, b, M, N, K, e, status);
+    if (pairs < 1) return cudaSuccess;
+    kern<<<2 * pairs, kPairThreads, SMEM, st>>>(args);
     return cudaGetLastError();
 }
 
@@ -884,13 +939,44 @@ bool tc_shape_ok(int64_t lda, int64_t ldb, int K, int64_t kz, const void* A, con
     return K >= 1;
 }
 
+// One problem of the pair kernel: 256 x 256 tiles, each CTA stages 128 rows of A
+// and 128 rows of B.
+static int pair_problem(PairProblem* P, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_t colsA,
+                        const __nv_bfloat16* B, int64_t ldb, int64_t rowsB, int64_t colsB, int M, int N, int K,
+                        const TcEpi& epi) {
+    if (!tc_shape_ok(lda, ldb, K, 0, A, B)) return fail(DBW_EALIGN, "tc_gemm: unsupported operand alignment");
+    if (!tc_make_map(&P->tmA, A, rowsA, colsA, lda, 64, BM) || !tc_make_map(&P->tmB, B, rowsB, colsB, ldb, 64, 128))
+        return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
+    P->M = M;
+    P->N = N;
+    P->K = K;
+    P->epi = epi;
+    return DBW_OK;
+}
+
+int tc_gemm_mean_dx(const TcOperands& g, const TcEpi& ge, const TcOperands& x, const TcEpi& xe, int* status,
+                    cudaStream_t st) {
+    PairArgs args{};
+    args.nprob = 2;
+    args.status = status;
+    int rc = pair_problem(&args.p[0], g.A, g.lda, g.rowsA, g.colsA, g.B, g.ldb, g.rowsB, g.colsB, g.M, g.N, g.K, ge);
+    if (rc) return rc;
+    rc = pair_problem(&args.p[1], x.A, x.lda, x.rowsA, x.colsA, x.B, x.ldb, x.rowsB, x.colsB, x.M, x.N, x.K, xe);
+    if (rc) return rc;
+    void* prof = profile_begin(PROF_GEMM, st, 0.0);
+    const cudaError_t e = launch_pair<TC_GBAR, TC_DX>(args, st);
+    profile_end(prof, st);
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "tc_gemm_mean_dx launch: %s", cudaGetErrorString(e));
+    return DBW_OK;
+}
+
 int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_t colsA, const __nv_bfloat16* B,
             int64_t ldb, int64_t rowsB, int64_t colsB, int M, int N, int K, int batch, int64_t kz, const TcEpi& epi,
             int* status, cudaStream_t st) {
-    if (!tc_shape_ok(lda, ldb, K, kz, A, B)) return fail(DBW_EALIGN, "tc_gemm: unsupported operand alignment");
-    CUtensorMap ta, tb;
     cudaError_t e = cudaSuccess;
     if (kind == TC_DW) {
+        if (!tc_shape_ok(lda, ldb, K, kz, A, B)) return fail(DBW_EALIGN, "tc_gemm: unsupported operand alignment");
+        CUtensorMap ta, tb;
         // K = the per-worker sample count: 64-deep blocks when it allows, else 32
         const int bk = (K % 64 == 0) ? 64 : 32;
         // algorithmic bytes: G written once (fp32), both bf16 operands read once
@@ -912,18 +998,20 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
         }
         profile_end(prof, st);
     } else {
-        // CTA pairs: 256 x 256 tiles, each CTA stages 128 rows of A and 128 rows of B
-        if (!tc_make_map(&ta, A, rowsA, colsA, lda, 64, BM) || !tc_make_map(&tb, B, rowsB, colsB, ldb, 64, 128))
-            return fail(DBW_ECUDA, "tc_gemm: cuTensorMapEncodeTiled failed");
+        PairArgs args{};
+        args.nprob = 1;
+        args.status = status;
+        const int rc = pair_problem(&args.p[0], A, lda, rowsA, colsA, B, ldb, rowsB, colsB, M, N, K, epi);
+        if (rc) return rc;
         void* prof = profile_begin(PROF_GEMM, st, 0.0);
         if (kind == TC_HIDDEN)
-            e = launch_pair<TC_HIDDEN>(ta, tb, M, N, K, epi, status, st);
+            e = launch_pair<TC_HIDDEN, TC_HIDDEN>(args, st);
         else if (kind == TC_LOGITS)
-            e = launch_pair<TC_LOGITS>(ta, tb, M, N, K, epi, status, st);
+            e = launch_pair<TC_LOGITS, TC_LOGITS>(args, st);
         else if (kind == TC_GBAR)
-            e = launch_pair<TC_GBAR>(ta, tb, M, N, K, epi, status, st);
+            e = launch_pair<TC_GBAR, TC_GBAR>(args, st);
         else
-            e = launch_pair<TC_DX>(ta, tb, M, N, K, epi, status, st);
+            e = launch_pair<TC_DX, TC_DX>(args, st);
         profile_end(prof, st);
     }
     if (e != cudaSuccess) return fail(DBW_ECUDA, "tc_gemm launch: %s", cudaGetErrorString(e));

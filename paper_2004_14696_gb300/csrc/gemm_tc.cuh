@@ -59,6 +59,22 @@ bool tc_make_map(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, 
 // True when tc_gemm can run this problem (alignment rules above).
 bool tc_shape_ok(int64_t lda, int64_t ldb, int K, int64_t kz, const void* A, const void* B);
 
+// Operands of one GEMM of tc_gemm_mean_dx (the same meaning as tc_gemm's arguments).
+struct TcOperands {
+    const __nv_bfloat16* A;
+    int64_t lda, rowsA, colsA;
+    const __nv_bfloat16* B;
+    int64_t ldb, rowsB, colsB;
+    int M, N, K;
+};
+
+// The mean-gradient GEMM (TC_GBAR, operands g, epilogue ge) and the input-gradient
+// GEMM (TC_DX, operands x, epilogue xe) of one layer in one launch: both read dZ_l
+// and neither writes what the other reads, so their tiles share the persistent
+// grid (those of the mean gradient first).  Same rules as tc_gemm.
+int tc_gemm_mean_dx(const TcOperands& g, const TcEpi& ge, const TcOperands& x, const TcEpi& xe, int* status,
+                    cudaStream_t st);
+
 // Per-worker squared gradient norms of one layer without forming the gradient
 // (the Gram identity ||D^T A||_F^2 = <D D^T, A A^T>_F, with the bias term
 // ||1^T D||^2 = sum of D D^T added):

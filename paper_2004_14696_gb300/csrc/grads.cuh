@@ -65,6 +65,8 @@ struct RxPlan {
     size_t off_pb[DBW_LMAX];           // fp64 [ceil(out_l / 256)]: pieces of ||g_t(b_l)||^2
     int npb[DBW_LMAX];
     size_t off_pg[DBW_LMAX];           // fp64 [(M / 32) * CT]: Gram pieces of ||g_j||^2
+    size_t off_dzT2;                   // bf16 [max width, M8]: second dZ^T buffer (the dX GEMM of a layer
+                                       // writes dZ_{l-1}^T while the mean-gradient GEMM reads dZ_l^T)
     size_t off_gpart;                  // fp32: partial Gram products of the K ranges (shared by the layers)
     size_t off_gcnt;                   // int32 [gram items]: per-item range counters, zeroed at the start of a call
     int ngcnt;

@@ -579,6 +579,7 @@ bool make_rx_plan(int L, const int32_t* widths, int n, int B, RxPlan* P) {
         P->off_pb[l] = take(static_cast<size_t>(P->npb[l]) * 8);
         P->off_pg[l] = take(static_cast<size_t>(g.M / 32) * P->CT * 8);
     }
+    P->off_dzT2 = take(static_cast<size_t>(maxout > g.widths[0] ? maxout : g.widths[0]) * P->t.M8 * 2);
     P->off_gpart = take(tc_gram_partial_floats(g.M, B) * 4);
     P->ngcnt = static_cast<int>(tc_gram_items(g.M, B));
     P->off_gcnt = take(static_cast<size_t>(P->ngcnt) * 4);
@@ -657,7 +658,11 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
     e = cudaGetLastError();
     if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
 
-    // backward: mean gradient + SGD step, bias, Gram norms, then dZ of the layer below
+    // backward: mean gradient + SGD step and dZ of the layer below (one launch), bias,
+    // Gram norms.  dZ_l^T alternates between two buffers: the dX GEMM writes dZ_{l-1}^T
+    // into one while the mean-gradient GEMM reads dZ_l^T from the other.
+    __nv_bfloat16* dzT[2] = {bf(T.off_dzT), bf(P.off_dzT2)};
+    int curT = 0;
     for (int l = L - 1; l >= 0; --l) {
         const int fin = g.widths[l], fout = g.widths[l + 1];
         TcEpi gb{};
@@ -669,8 +674,24 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
         gb.pieces = f64(P.off_pw[l]);
         gb.kdev = kdev;
         gb.kmul = B;
-        int rc = tc_gemm(TC_GBAR, bf(T.off_dzT), T.M8, fout, M, bf(T.off_actT[l]), T.M8, fin, M, fout, fin, M, 1, 0,
-                         gb, status, st);
+        const TcOperands go{dzT[curT], T.M8, fout, M, bf(T.off_actT[l]), T.M8, fin, M, fout, fin, M};
+        int rc;
+        if (l > 0) {
+            TcEpi ex{};
+            ex.act = bf(T.off_act[l]);
+            ex.ldact = T.ldact[l];
+            ex.out = bf(T.off_dz[cur ^ 1]);
+            ex.ldo = T.ldz;
+            ex.outT = dzT[curT ^ 1];
+            ex.ldT = T.M8;
+            ex.kdev = kdev;
+            ex.kmul = B;
+            const TcOperands xo{bf(T.off_dz[cur]), T.ldz, M, fout, bf(T.off_wt[l]), T.ldwt[l], fin, fout, M, fin, fout};
+            rc = tc_gemm_mean_dx(go, gb, xo, ex, status, st);
+        } else {
+            rc = tc_gemm(TC_GBAR, go.A, go.lda, go.rowsA, go.colsA, go.B, go.ldb, go.rowsB, go.colsB, go.M, go.N, go.K,
+                         1, 0, gb, status, st);
+        }
         if (rc) return rc;
         bias_rows_kernel<<<dim3((fout + 255) / 256, (M + 255) / 256), 256, 0, st>>>(bf(T.off_dz[cur]), T.ldz, fout,
                                                                                    B, kdev, bpart);
@@ -682,19 +703,8 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
                      gpart, gcnt, status, st);
         if (rc) return rc;
         if (l > 0) {
-            TcEpi ex{};
-            ex.act = bf(T.off_act[l]);
-            ex.ldact = T.ldact[l];
-            ex.out = bf(T.off_dz[cur ^ 1]);
-            ex.ldo = T.ldz;
-            ex.outT = bf(T.off_dzT);
-            ex.ldT = T.M8;
-            ex.kdev = kdev;
-            ex.kmul = B;
-            rc = tc_gemm(TC_DX, bf(T.off_dz[cur]), T.ldz, M, fout, bf(T.off_wt[l]), T.ldwt[l], fin, fout, M, fin,
-                         fout, 1, 0, ex, status, st);
-            if (rc) return rc;
             cur ^= 1;
+            curT ^= 1;
         }
     }
     FinishArgs fa{};
