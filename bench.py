@@ -363,7 +363,7 @@ def _run_dbw(args, rank, world, local_rank, clk):
     tensor = None
     if gm_launches:
         tf = tc_flop * K / (gm_ms * 1e-3) / 1e12
-        tensor = {"kernel": "tc_gemm_persistent_kernel (forward + input-gradient GEMMs, in dbw_worker_grads)",
+        tensor = {"kernel": "tc_gemm_pair_kernel (forward + input-gradient GEMMs, in dbw_worker_grads)",
                   "bound": "tensor", "achieved": tf, "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s",
                   "frac": tf / pk["bf16_tflops_sustained"], "traffic": None,
                   "algorithmic_flop_per_step": tc_flop, "ms_per_step": gm_ms / K,
@@ -404,7 +404,7 @@ def _run_dbw(args, rank, world, local_rank, clk):
         gms, gl = rx.pop("_gemm")
         if gl:
             tf = flop / (gms * 1e-3) / 1e12
-            rx["roofline"] = {"kernel": "tc_gemm_persistent_kernel (forward, mean-gradient and input-gradient "
+            rx["roofline"] = {"kernel": "tc_gemm_pair_kernel (forward, mean-gradient and input-gradient "
                                         "GEMMs, in dbw_received_grads_update)",
                               "bound": "tensor", "achieved": tf, "peak": pk["bf16_tflops_sustained"],
                               "unit": "TFLOP/s", "frac": tf / pk["bf16_tflops_sustained"], "traffic": None,
