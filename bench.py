@@ -49,10 +49,11 @@ AGG_TRAFFIC = {"ratio_to_algorithmic": 793.76e6 / 800.0e6, "source_sha256": "415
                "case": "n=64 d=4e6 k=48"}
 # dram bytes (read + write) of the per-worker weight-gradient launches of one
 # full-size step (ncu on mlp4096x3-1000_n256_B32, profiles/tc_dw_kernel_mlp4096_ncu.md):
-# 4.2130 + 17.2560 + 17.2543 + 17.2546 GB against 4.2778 + 3 x 17.3141 GB algorithmic;
+# 4.2130 + 17.2599 + 17.2596 + 17.2583 GB against 4.2778 + 3 x 17.3141 GB algorithmic;
 # keyed to the dW kernel's own source (dw_source_sha).
-DW_TRAFFIC = {"ratio_to_algorithmic": (4.2130 + 17.2560 + 17.2543 + 17.2546) / (4.2778 + 3 * 17.3141),
-              "source_sha256": "9a7ee52ced946ba0dc44c00873f852f1e90ae35e2f879b1d4e6915a983e936fe", "case": "mlp4096x3-1000_n256_B32, one step"}
+DW_TRAFFIC = {"ratio_to_algorithmic": (4.2130 + 17.2599 + 17.2596 + 17.2583) / (4.2778 + 3 * 17.3141),
+              "source_sha256": "49652b56fb1338974566dcb78b1b940bb43688a603dfa846f820898c31d62839",
+              "case": "mlp4096x3-1000_n256_B32, one step"}
 
 
 def parse():
