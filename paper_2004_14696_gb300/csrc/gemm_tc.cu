@@ -73,9 +73,19 @@ __device__ __forceinline__ void epilogue_chunk(const TcEpi& e, int z, int row, i
 // step, the layer input for the ReLU mask) are issued one chunk ahead, so that
 // their latency overlaps the previous chunk's work.
 
-// bf16 activation chunk -> out (row-major) and, when asked, outT (transposed: the 32
-// lanes of a warp hold 32 consecutive rows, so each store covers 64 contiguous bytes).
-__device__ __forceinline__ void store_act_chunk(const TcEpi& e, int row, int nb, int N, const float (&x)[32]) {
+// Per epilogue warp: a 32 x 32 bf16 chunk, transposed ([column][row], rows padded to 40
+// elements), between TMEM and the transposed copy.
+constexpr int kStageLd = 40;
+constexpr int kStageBytes = 32 * kStageLd * 2;
+
+// bf16 activation chunk -> out (row-major) and, when asked, outT (transposed).  The
+// lanes of a warp hold 32 consecutive rows (row = row0 + lane; M is a multiple of 32,
+// so a warp's rows are all inside or all outside the matrix); the transposed copy goes
+// through the warp's staging chunk ``stg`` so that each global store writes 16 bytes
+// and four lanes cover 64 contiguous bytes of one transposed row.
+__device__ __forceinline__ void store_act_chunk(const TcEpi& e, int row, int nb, int N, const float (&x)[32],
+                                                __nv_bfloat16* stg) {
+    const int lane = threadIdx.x & 31;
     __nv_bfloat16* op = e.out + static_cast<int64_t>(row) * e.ldo + nb;
     if (nb + 32 <= N && ((reinterpret_cast<uintptr_t>(op) & 15u) == 0)) {
 #pragma unroll
@@ -94,13 +104,32 @@ __device__ __forceinline__ void store_act_chunk(const TcEpi& e, int row, int nb,
     }
     if (e.outT) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j)
-            if (nb + j < N) e.outT[static_cast<int64_t>(nb + j) * e.ldT + row] = __float2bfloat16_rn(x[j]);
+        for (int j = 0; j < 32; ++j) stg[j * kStageLd + lane] = __float2bfloat16_rn(x[j]);
+        __syncwarp();
+        const int row0 = row - lane;
+        const bool vec = ((reinterpret_cast<uintptr_t>(e.outT) & 15u) == 0) && e.ldT % 8 == 0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int idx = i * 32 + lane;
+            const int j = idx >> 2, p = idx & 3;   // transposed row nb + j, rows row0 + 8p .. +7
+            if (nb + j < N) {
+                __nv_bfloat16* dst = e.outT + static_cast<int64_t>(nb + j) * e.ldT + row0 + 8 * p;
+                const __nv_bfloat16* src = stg + j * kStageLd + 8 * p;
+                if (vec) {
+                    *reinterpret_cast<uint4*>(dst) = *reinterpret_cast<const uint4*>(src);
+                } else {
+#pragma unroll
+                    for (int t = 0; t < 8; ++t) dst[t] = src[t];
+                }
+            }
+        }
+        __syncwarp();
     }
 }
 
 // TC_HIDDEN: A_l = ReLU(Z_l + b_l) in bf16.
-__device__ __forceinline__ void hidden_cols(const TcEpi& e, int row, int nb0, int M, int N, uint32_t taddr) {
+__device__ __forceinline__ void hidden_cols(const TcEpi& e, int row, int nb0, int M, int N, uint32_t taddr,
+                                            __nv_bfloat16* stg) {
 #pragma unroll 1
     for (int c = 0; c < 4; ++c) {
         const int nb = nb0 + 32 * c;
@@ -115,13 +144,14 @@ __device__ __forceinline__ void hidden_cols(const TcEpi& e, int row, int nb0, in
             const float v = u2f(r[j]) + (nb + j < N ? __ldg(e.bias + nb + j) : 0.f);
             x[j] = v > 0.f ? v : 0.f;
         }
-        store_act_chunk(e, row, nb, N, x);
+        store_act_chunk(e, row, nb, N, x, stg);
     }
 }
 
 // TC_DX: dZ_{l-1} = (dZ_l W_l) * 1[A_{l-1} > 0] in bf16; ``avec``: the act rows allow
 // 16-byte loads.
-__device__ __forceinline__ void dx_cols(const TcEpi& e, int row, int nb0, int M, int N, uint32_t taddr, bool avec) {
+__device__ __forceinline__ void dx_cols(const TcEpi& e, int row, int nb0, int M, int N, uint32_t taddr, bool avec,
+                                        __nv_bfloat16* stg) {
     const bool rowok = row < M;
     const __nv_bfloat16* ap = e.act + static_cast<int64_t>(row) * e.ldact + nb0;
     uint4 nxt[4];
@@ -158,7 +188,7 @@ __device__ __forceinline__ void dx_cols(const TcEpi& e, int row, int nb0, int M,
             for (int j = 0; j < 32; ++j)
                 x[j] = (nb + j < N) ? u2f(r[j]) * (__bfloat162float(ap[32 * c + j]) > 0.f ? 1.f : 0.f) : 0.f;
         }
-        store_act_chunk(e, row, nb, N, x);
+        store_act_chunk(e, row, nb, N, x, stg);
     }
 }
 
@@ -415,7 +445,7 @@ __device__ __forceinline__ PairShape pair_shape(const PairProblem& P) {
 // Epilogue of one tile for problem kind KIND (one thread: one row, 128 columns).
 template <int KIND>
 __device__ __forceinline__ void pair_epilogue(const PairProblem& P, const PairShape& S, long long t, int rank, int q,
-                                              int h, int lane, uint32_t taddr) {
+                                              int h, int lane, uint32_t taddr, __nv_bfloat16* stg) {
     constexpr int BN = 256;
     const TcEpi& epi = P.epi;
     const int nt = static_cast<int>(t % S.nt_n);
@@ -433,9 +463,9 @@ __device__ __forceinline__ void pair_epilogue(const PairProblem& P, const PairSh
         if (lane == 0 && msub < S.msub_n) epi.pieces[(static_cast<long long>(msub) * S.nt_n + nt) * 8 + h * 4 + q] = sq;
     } else if constexpr (KIND == TC_DX) {
         const bool avec = ((reinterpret_cast<uintptr_t>(epi.act) & 15u) == 0) && epi.ldact % 8 == 0;
-        dx_cols(epi, row, nb0, P.M, P.N, taddr, avec);
+        dx_cols(epi, row, nb0, P.M, P.N, taddr, avec, stg);
     } else if constexpr (KIND == TC_HIDDEN) {
-        hidden_cols(epi, row, nb0, P.M, P.N, taddr);
+        hidden_cols(epi, row, nb0, P.M, P.N, taddr, stg);
     } else {
 #pragma unroll 1
         for (int c = 0; c < 4; ++c) {
@@ -465,6 +495,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     uint64_t* tempty_bar = tfull_bar + 2;        // [2]
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty_bar + 2);
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+    // epilogue warps' transposing chunks, after the 256 bytes of barriers
+    __nv_bfloat16* staging = reinterpret_cast<__nv_bfloat16*>(smem + STAGES * STAGE_BYTES + 256);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t rank = cluster_rank();
@@ -576,6 +608,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     } else if (warp >= 2) {
         // ---------------- epilogue (both CTAs): 128-row sub-tile msub, lane quarter q, column half h
         const int q = warp & 3, h = (warp - 2) >> 2;
+        __nv_bfloat16* stg = staging + (warp - 2) * (kStageBytes / 2);
         int i = 0;
         for (long long t = pair; t < total; t += npairs, ++i) {
             const int acc = i & 1;
@@ -590,9 +623,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
             const uint32_t taddr = tmem + static_cast<uint32_t>(acc * BN + h * (BN / 2)) +
                                    (static_cast<uint32_t>(q * 32) << 16);
             if (t < S0.tiles)
-                pair_epilogue<KIND0>(args.p[0], S0, t, static_cast<int>(rank), q, h, lane, taddr);
+                pair_epilogue<KIND0>(args.p[0], S0, t, static_cast<int>(rank), q, h, lane, taddr, stg);
             else
-                pair_epilogue<KIND1>(args.p[1], S1, t - S0.tiles, static_cast<int>(rank), q, h, lane, taddr);
+                pair_epilogue<KIND1>(args.p[1], S1, t - S0.tiles, static_cast<int>(rank), q, h, lane, taddr,
+                                     stg);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_remote(map_to_rank(smem_u32(tempty_bar + acc), 0));
@@ -867,7 +901,7 @@ int pair_slots(Kern kern, int smem) {
 template <int KIND0, int KIND1>
 cudaError_t launch_pair(const PairArgs& args, cudaStream_t st) {
     constexpr int STAGES = DBW_PAIR_STAGES;
-    constexpr int SMEM = STAGES * (2 * BM * 64 * 2) + 256 + 1024;
+    constexpr int SMEM = STAGES * (2 * BM * 64 * 2) + 256 + 8 * kStageBytes + 1024;
     static_assert(SMEM <= 227 * 1024, "pair ring does not fit in shared memory");
     auto kern = tc_gemm_pair_kernel<KIND0, KIND1, STAGES>;
     cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
