@@ -258,3 +258,61 @@ def psw_margin(st, lr, beta, T):
     if st.t >= 2 and st.k_last < st.n:
         gaps.append(abs(st.F_last - beta * st.F_prev) / abs(st.F_last))
     return min(gaps)
+
+
+@pytest.mark.parametrize("n", [96, 200])
+def test_fit_on_planted_tables(n):
+    """Eq. (17) on cell tables written straight into the state, shaped so that the split
+    chains pool across their parts: group rows whose cell means fall along the whole row
+    (one block absorbs every part), rise (nothing pools), or zig-zag, with random counts;
+    rows outside the group feed only the pooled column means.  Against the oracle's fit
+    of the same table."""
+    rng = np.random.default_rng(n)
+    psw = dbw.new_psw(n)
+    ps = P.psw_init(n)
+    unit = 2.0 ** -32
+    sums = np.zeros((n, n), np.uint64)
+    cnts = np.zeros((n, n), np.int32)
+    group = sorted(rng.choice(np.arange(2, n - 2), size=5, replace=False).tolist())
+    shapes = ["fall", "rise", "zigzag", "fall", "random"]
+    for h, shape in zip(group, shapes):           # 1-based row h, observed prefix 1..M_h
+        M = int(rng.integers(h, n + 1))
+        i = np.arange(M)
+        if shape == "fall":
+            mean = 50.0 - 40.0 * i / M
+        elif shape == "rise":
+            mean = 5.0 + 40.0 * i / M
+        elif shape == "zigzag":
+            mean = 20.0 + 10.0 * (i % 7) - 0.05 * i
+        else:
+            mean = rng.uniform(1.0, 40.0, size=M)
+        c = rng.integers(1, 6, size=M)
+        q = np.round(mean * c / unit)             # cell sums in 2^-32 units, as the clock stores them
+        sums[h - 1, :M] = q.astype(np.uint64)
+        cnts[h - 1, :M] = c
+    for h in rng.choice([r for r in range(1, n) if r not in group], size=4, replace=False):
+        M = int(rng.integers(1, h))                # below the diagonal: not in the fitted group
+        c = rng.integers(1, 4, size=M)
+        sums[h - 1, :M] = np.round(rng.uniform(1.0, 40.0, size=M) * c / unit).astype(np.uint64)
+        cnts[h - 1, :M] = c
+    import ctypes
+    hdr = dbw.PswHeader.from_buffer_copy(psw[:ctypes.sizeof(dbw.PswHeader)].cpu().numpy().tobytes())
+    assert hdr.n == n
+    psw[hdr.off_sum:hdr.off_sum + 8 * n * n] = torch.from_numpy(sums.reshape(-1).view(np.uint8)).cuda()
+    psw[hdr.off_cnt:hdr.off_cnt + 4 * n * n] = torch.from_numpy(cnts.reshape(-1).view(np.uint8)).cuda()
+    ps.sums[1:, 1:] = sums.astype(np.float64) * unit
+    ps.cnts[1:, 1:] = cnts
+    T = torch.empty(n, dtype=torch.float64, device="cuda")
+    dbw.dbw_psw_estimate(psw, n, T, tol=1e-6, max_sweeps=200000)
+    torch.cuda.synchronize()
+    g = dbw.read_psw(psw, n)
+    assert not (g["flags"] & dbw.PSW_NOT_CONVERGED)
+    ref = np.array(P.time_estimates(ps, tol=1e-11))
+    got = T.cpu().numpy()
+    assert np.all(np.abs(got - ref) <= 2e-5 * np.max(np.abs(ref))), np.max(np.abs(got - ref))
+    # the fitted group cells themselves
+    H, fit, _ = P.solve(ps, tol=1e-11)
+    scale = max(abs(v) for v in fit.values())
+    for (h, i), v in fit.items():
+        assert abs(float(g["x"][h - 1, i - 1]) - v) <= 2e-5 * scale, (h, i, float(g["x"][h - 1, i - 1]), v)
+
