@@ -305,8 +305,8 @@ size_t dbw_received_partials_bytes(int n);
  *     forward / backward GEMMs run over those k B rows (under push-and-interrupt,
  *     Sect. 3, the other workers' gradients are never used);
  *   Eqs. (3)-(4): g_t(W_l) = (1/k) dZ_l^T A_{l-1} over the k B stacked rows, one
- *     GEMM with K = k B whose epilogue applies w -= lr g_t; the bias part is the
- *     mean of the per-worker column sums of dZ_l;
+ *     GEMM with K = k B whose epilogue applies w -= lr g_t; the bias part is
+ *     (1/k) times the column sums of dZ_l over the k B rows;
  *   ||g_j||^2 of every received worker from two B x B Gram matrices per layer,
  *     ||dZ_j^T A_j||^2 + ||1^T dZ_j||^2 = <dZ_j dZ_j^T, A_j A_j^T + 1 1^T>
  *     (never forming g_j);
