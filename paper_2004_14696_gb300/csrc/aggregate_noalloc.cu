@@ -86,6 +86,7 @@ using namespace dbw;
 
 extern "C" int dbw_aggregate_update_noalloc(const float* G, int64_t ld, int n, int64_t d, const uint8_t* mask,
                                             float lr, float* w, float* gbar, double* sums_out, void* stream) {
+    Call call("dbw_aggregate_update_noalloc", as_stream(stream));
     if (!G || !mask || !w || !sums_out)
         return fail(DBW_EINVAL, "dbw_aggregate_update_noalloc: NULL pointer argument");
     if (n < 1 || n > DBW_NMAX)
@@ -113,5 +114,5 @@ extern "C" int dbw_aggregate_update_noalloc(const float* G, int64_t ld, int n, i
     reduce_to_sums_kernel<<<n + 2, kRed, 0, st>>>(partials, n, sums_out);
     e = cudaGetLastError();
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_aggregate_update_noalloc: %s", cudaGetErrorString(e));
-    return DBW_OK;
+    return call.done(DBW_OK);
 }

@@ -1,8 +1,10 @@
 // extern "C" entry points of libdbw (declared in include/dbw.h): host-side
 // argument checks, then launches on the caller's stream.  No entry point
 // allocates device memory.
+#include <nvtx3/nvToolsExt.h>
 #include <stdarg.h>
 #include <stdio.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include "common.cuh"
@@ -40,6 +42,24 @@ int sm_count() {
     if (dev < 0 || dev >= 64) return device_sm_count_uncached(dev);
     if (cache[dev] == 0) cache[dev] = device_sm_count_uncached(dev);
     return cache[dev];
+}
+
+Call::Call(const char* name, cudaStream_t st) : name_(name), st_(st) { nvtxRangePushA(name); }
+
+Call::~Call() { nvtxRangePop(); }
+
+int Call::done(int rc) {
+    static const bool sync = [] {
+        const char* v = getenv("DBW_DEBUG_SYNC");
+        return v && v[0] == '1';
+    }();
+    if (rc != DBW_OK || !sync) return rc;
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st_, &cap) != cudaSuccess || cap != cudaStreamCaptureStatusNone) return rc;
+    const cudaError_t e = cudaStreamSynchronize(st_);
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s (reported by the debug synchronisation)", name_,
+                                      cudaGetErrorString(e));
+    return rc;
 }
 
 int check_device() {
@@ -94,6 +114,7 @@ int dbw_worker_grads(int num_layers, const int32_t* widths, int prec, const floa
                      int64_t S, const int32_t* labels, const int32_t* idx, int n, int B, float* G, int64_t ld,
                      float* loss, void* ws, size_t ws_bytes, void* stream) {
     g_err[0] = 0;
+    Call call("dbw_worker_grads", as_stream(stream));
     if (!widths || !w || !pool || !labels || !idx || !G || !loss || !ws)
         return fail(DBW_EINVAL, "dbw_worker_grads: NULL pointer argument");
     if (S < 1) return fail(DBW_EINVAL, "dbw_worker_grads: S must be >= 1");
@@ -104,13 +125,14 @@ int dbw_worker_grads(int num_layers, const int32_t* widths, int prec, const floa
         return fail(DBW_EALIGN, "dbw_worker_grads: widths[0] must be a multiple of 4");
     int rc = check_device();
     if (rc) return rc;
-    return launch_worker_grads(num_layers, widths, prec, w, d, pool, S, labels, idx, n, B, G, ld, loss, ws, ws_bytes,
-                               as_stream(stream));
+    return call.done(launch_worker_grads(num_layers, widths, prec, w, d, pool, S, labels, idx, n, B, G, ld, loss,
+                                         ws, ws_bytes, as_stream(stream)));
 }
 
 int dbw_select_fastest(const double* times, int n, const int32_t* b, int32_t* order, uint8_t* mask, double* tsorted,
                        int32_t* k_out, void* stream) {
     g_err[0] = 0;
+    Call call("dbw_select_fastest", as_stream(stream));
     if (!times || !b || !order || !mask || !tsorted)
         return fail(DBW_EINVAL, "dbw_select_fastest: NULL pointer argument");
     if (n < 1 || n > DBW_NMAX) return fail(DBW_EINVAL, "dbw_select_fastest: n must be in [1, %d]", DBW_NMAX);
@@ -118,7 +140,7 @@ int dbw_select_fastest(const double* times, int n, const int32_t* b, int32_t* or
     if (rc) return rc;
     cudaError_t e = launch_select(times, n, b, order, mask, tsorted, k_out, as_stream(stream));
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_select_fastest: %s", cudaGetErrorString(e));
-    return DBW_OK;
+    return call.done(DBW_OK);
 }
 
 size_t dbw_aggregate_partials_bytes(int n, int64_t d) {
@@ -129,6 +151,7 @@ size_t dbw_aggregate_partials_bytes(int n, int64_t d) {
 int dbw_aggregate_update(const float* G, int64_t ld, int n, int64_t d, const uint8_t* mask, float lr, float* w,
                          float* gbar, double* partials, size_t partials_bytes, void* stream) {
     g_err[0] = 0;
+    Call call("dbw_aggregate_update", as_stream(stream));
     if (!G || !mask || !w || !partials) return fail(DBW_EINVAL, "dbw_aggregate_update: NULL pointer argument");
     if (n < 1 || n > DBW_NMAX) return fail(DBW_EINVAL, "dbw_aggregate_update: n must be in [1, %d]", DBW_NMAX);
     if (d < 1) return fail(DBW_EINVAL, "dbw_aggregate_update: d must be >= 1");
@@ -142,7 +165,7 @@ int dbw_aggregate_update(const float* G, int64_t ld, int n, int64_t d, const uin
         return fail(DBW_EINVAL, "dbw_aggregate_update: partials %zu bytes < %zu needed", partials_bytes, g.bytes);
     cudaError_t e = launch_aggregate(G, ld, n, d, mask, lr, w, gbar, partials, g, as_stream(stream));
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_aggregate_update: %s", cudaGetErrorString(e));
-    return DBW_OK;
+    return call.done(DBW_OK);
 }
 
 size_t dbw_received_grads_workspace_bytes(int num_layers, const int32_t* widths, int n, int B, int prec) {
@@ -160,6 +183,7 @@ int dbw_received_grads_update(int num_layers, const int32_t* widths, int prec, f
                               float lr, float* gbar, float* loss, double* partials, size_t partials_bytes, void* ws,
                               size_t ws_bytes, void* stream) {
     g_err[0] = 0;
+    Call call("dbw_received_grads_update", as_stream(stream));
     if (!widths || !w || !pool || !labels || !idx || !mask || !loss || !partials || !ws)
         return fail(DBW_EINVAL, "dbw_received_grads_update: NULL pointer argument");
     if (S < 1) return fail(DBW_EINVAL, "dbw_received_grads_update: S must be >= 1");
@@ -174,12 +198,13 @@ int dbw_received_grads_update(int num_layers, const int32_t* widths, int prec, f
         return fail(DBW_EALIGN, "dbw_received_grads_update: widths[0] must be a multiple of 4");
     int rc = check_device();
     if (rc) return rc;
-    return launch_received_grads(num_layers, widths, prec, w, d, pool, S, labels, idx, n, B, mask, lr, gbar, loss,
-                                 partials, ws, ws_bytes, as_stream(stream));
+    return call.done(launch_received_grads(num_layers, widths, prec, w, d, pool, S, labels, idx, n, B, mask, lr,
+                                           gbar, loss, partials, ws, ws_bytes, as_stream(stream)));
 }
 
 int dbw_state_init(dbw_state* state, int n, int D, void* stream) {
     g_err[0] = 0;
+    Call call("dbw_state_init", as_stream(stream));
     if (!state) return fail(DBW_EINVAL, "dbw_state_init: NULL state");
     if (n < 1 || n > DBW_NMAX) return fail(DBW_EINVAL, "dbw_state_init: n must be in [1, %d]", DBW_NMAX);
     if (D < 1 || D > DBW_DMAX) return fail(DBW_EINVAL, "dbw_state_init: D must be in [1, %d]", DBW_DMAX);
@@ -188,12 +213,13 @@ int dbw_state_init(dbw_state* state, int n, int D, void* stream) {
     if (rc) return rc;
     cudaError_t e = launch_state_init(state, n, D, as_stream(stream));
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_state_init: %s", cudaGetErrorString(e));
-    return DBW_OK;
+    return call.done(DBW_OK);
 }
 
 int dbw_grad_stats(const double* partials, int n, const uint8_t* mask, const float* loss, const double* tsorted,
                    double lr, dbw_state* state, double* stats_out, double* row_sqnorm, void* stream) {
     g_err[0] = 0;
+    Call call("dbw_grad_stats", as_stream(stream));
     if (!partials || !mask || !loss || !tsorted || !state)
         return fail(DBW_EINVAL, "dbw_grad_stats: NULL pointer argument");
     if (n < 1 || n > DBW_NMAX) return fail(DBW_EINVAL, "dbw_grad_stats: n must be in [1, %d]", DBW_NMAX);
@@ -204,12 +230,13 @@ int dbw_grad_stats(const double* partials, int n, const uint8_t* mask, const flo
     cudaError_t e = launch_grad_stats(partials, n, mask, loss, tsorted, lr, state, stats_out, row_sqnorm,
                                       as_stream(stream));
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_grad_stats: %s", cudaGetErrorString(e));
-    return DBW_OK;
+    return call.done(DBW_OK);
 }
 
 int dbw_choose_b(dbw_state* state, double lr, double beta, int flags, int32_t* b_out, double* ratio_out,
                  void* stream) {
     g_err[0] = 0;
+    Call call("dbw_choose_b", as_stream(stream));
     if (!state || !b_out) return fail(DBW_EINVAL, "dbw_choose_b: NULL pointer argument");
     if (!(lr > 0.0)) return fail(DBW_EINVAL, "dbw_choose_b: lr must be > 0");
     if (!(beta >= 1.0)) return fail(DBW_EINVAL, "dbw_choose_b: beta must be >= 1");
@@ -219,12 +246,13 @@ int dbw_choose_b(dbw_state* state, double lr, double beta, int flags, int32_t* b
     if (rc) return rc;
     cudaError_t e = launch_choose_b(state, lr, beta, flags, b_out, ratio_out, nullptr, as_stream(stream));
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_choose_b: %s", cudaGetErrorString(e));
-    return DBW_OK;
+    return call.done(DBW_OK);
 }
 
 int dbw_choose_b_times(dbw_state* state, const double* T_hat, double lr, double beta, int flags, int32_t* b_out,
                        double* ratio_out, void* stream) {
     g_err[0] = 0;
+    Call call("dbw_choose_b_times", as_stream(stream));
     if (!state || !T_hat || !b_out) return fail(DBW_EINVAL, "dbw_choose_b_times: NULL pointer argument");
     if (!(lr > 0.0)) return fail(DBW_EINVAL, "dbw_choose_b_times: lr must be > 0");
     if (!(beta >= 1.0)) return fail(DBW_EINVAL, "dbw_choose_b_times: beta must be >= 1");
@@ -234,7 +262,7 @@ int dbw_choose_b_times(dbw_state* state, const double* T_hat, double lr, double 
     if (rc) return rc;
     cudaError_t e = launch_choose_b(state, lr, beta, flags, b_out, ratio_out, T_hat, as_stream(stream));
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_choose_b_times: %s", cudaGetErrorString(e));
-    return DBW_OK;
+    return call.done(DBW_OK);
 }
 
 size_t dbw_psw_bytes(int n) {
@@ -251,35 +279,39 @@ static int psw_args(const char* what, const void* psw, int n) {
 
 int dbw_psw_init(void* psw, int n, void* stream) {
     g_err[0] = 0;
+    Call call("dbw_psw_init", as_stream(stream));
     int rc = psw_args("dbw_psw_init", psw, n);
     if (rc) return rc;
     cudaError_t e = launch_psw_init(psw, n, as_stream(stream));
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_psw_init: %s", cudaGetErrorString(e));
-    return DBW_OK;
+    return call.done(DBW_OK);
 }
 
 int dbw_psw_arrivals(const void* psw, int n, const double* omega, double* arrivals, void* stream) {
     g_err[0] = 0;
+    Call call("dbw_psw_arrivals", as_stream(stream));
     if (!omega || !arrivals) return fail(DBW_EINVAL, "dbw_psw_arrivals: NULL pointer argument");
     int rc = psw_args("dbw_psw_arrivals", psw, n);
     if (rc) return rc;
     cudaError_t e = launch_psw_arrivals(psw, n, omega, arrivals, as_stream(stream));
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_psw_arrivals: %s", cudaGetErrorString(e));
-    return DBW_OK;
+    return call.done(DBW_OK);
 }
 
 int dbw_psw_record(void* psw, int n, const int32_t* order, const double* tsorted, const int32_t* k, void* stream) {
     g_err[0] = 0;
+    Call call("dbw_psw_record", as_stream(stream));
     if (!order || !tsorted || !k) return fail(DBW_EINVAL, "dbw_psw_record: NULL pointer argument");
     int rc = psw_args("dbw_psw_record", psw, n);
     if (rc) return rc;
     cudaError_t e = launch_psw_record(psw, n, order, tsorted, k, as_stream(stream));
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_psw_record: %s", cudaGetErrorString(e));
-    return DBW_OK;
+    return call.done(DBW_OK);
 }
 
 int dbw_psw_estimate(void* psw, int n, double tol, int max_sweeps, double* T_hat, void* stream) {
     g_err[0] = 0;
+    Call call("dbw_psw_estimate", as_stream(stream));
     if (!T_hat) return fail(DBW_EINVAL, "dbw_psw_estimate: NULL T_hat");
     if (!(tol > 0.0)) return fail(DBW_EINVAL, "dbw_psw_estimate: tol must be > 0");
     if (max_sweeps < 1) return fail(DBW_EINVAL, "dbw_psw_estimate: max_sweeps must be >= 1");
@@ -287,7 +319,7 @@ int dbw_psw_estimate(void* psw, int n, double tol, int max_sweeps, double* T_hat
     if (rc) return rc;
     cudaError_t e = launch_psw_estimate(psw, n, tol, max_sweeps, T_hat, as_stream(stream));
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_psw_estimate: %s", cudaGetErrorString(e));
-    return DBW_OK;
+    return call.done(DBW_OK);
 }
 
 }  // extern "C"

@@ -18,6 +18,25 @@ int sm_count();
 // DBW_OK if the current device is sm_103 (compute capability 10.3), else DBW_EUNSUPPORTED.
 int check_device();
 
+// One C-ABI call: an NVTX range named after the entry point (seen by timeline tools,
+// a no-op otherwise) and, with DBW_DEBUG_SYNC=1 in the environment, a
+// synchronisation of the call's stream before it returns, so that an asynchronous
+// fault is reported by the call that launched it (skipped while the stream is being
+// captured into a graph).
+class Call {
+public:
+    Call(const char* name, cudaStream_t st);
+    ~Call();
+    Call(const Call&) = delete;
+    Call& operator=(const Call&) = delete;
+    // rc, or DBW_ECUDA when the debug synchronisation reports an error.
+    int done(int rc);
+
+private:
+    const char* name_;
+    cudaStream_t st_;
+};
+
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 inline bool aligned256(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 255u) == 0; }
 inline cudaStream_t as_stream(void* s) { return reinterpret_cast<cudaStream_t>(s); }

@@ -165,3 +165,37 @@ def test_graph_replay_is_the_same_iteration(form):
         assert torch.equal(eager.b, graphed.b) and torch.equal(eager.mask, graphed.mask), t
         if form == "psw":
             assert torch.equal(eager.psw, graphed.psw), t
+
+
+def test_debug_sync_mode():
+    """DBW_DEBUG_SYNC=1 (read once per process): every call synchronises its stream
+    before returning, except while the stream is being captured into a graph; eager
+    steps and a captured, replayed iteration both still run clean."""
+    import os
+    import subprocess
+    import sys
+    code = r'''
+import torch
+import __graft_entry__
+__graft_entry__.build()
+from paper_2004_14696_gb300 import workloads
+from paper_2004_14696_gb300.pipeline import Iteration
+wl = workloads.Workload(key="dbgsync", widths=(256, 128, 10), n=8, B=32, prec=workloads.PREC_BF16, S=300,
+                        feature_dist="normal", time_model="pareto", time_params={"alpha": 2.0}, lr=0.01,
+                        seed_offset=96)
+for received in (False, True):
+    it = Iteration(wl, received=received)
+    for t in range(3):
+        it.load_inputs(t)
+        it.step()
+    it.capture()
+    it.load_inputs(3)
+    it.replay()
+    torch.cuda.synchronize()
+    assert int(it.ws[:4].view(torch.int32).item()) == 0
+print("ok")
+'''
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ, DBW_DEBUG_SYNC="1", PYTHONPATH=root)
+    out = subprocess.run([sys.executable, "-c", code], cwd=root, env=env, capture_output=True, text=True, timeout=600)
+    assert out.returncode == 0 and out.stdout.strip().endswith("ok"), out.stderr[-3000:]
