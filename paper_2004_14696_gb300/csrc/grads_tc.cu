@@ -201,6 +201,7 @@ __global__ void __launch_bounds__(256) softmax_xent_ld_kernel(const float* __res
     if (threadIdx.x == 0) bad_s = 0;
     __syncthreads();
     const float invB = 1.0f / static_cast<float>(B);
+    constexpr int kRegs = 32;   // logits a lane keeps in registers: rows of up to 1024 classes in one read
     for (int r = warp; r < B; r += nw) {
         const int64_t row = static_cast<int64_t>(i) * B + r;
         const int64_t sidx = idx[static_cast<int64_t>(worker) * B + r];
@@ -208,19 +209,48 @@ __global__ void __launch_bounds__(256) softmax_xent_ld_kernel(const float* __res
         if (sidx >= 0 && sidx < S) y = labels[sidx];
         const bool bad = (y < 0 || y >= C);
         const float* z = logits + row * ldl;
-        float mx = -INFINITY;
-        for (int c = lane; c < C; c += 32) mx = fmaxf(mx, z[c]);
+        float mx = -INFINITY, se = 0.f;
+        if (C <= 32 * kRegs) {
+            // the row is read once: max, sum of exponentials and dZ from registers
+            float v[kRegs];
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-        float se = 0.f;
-        for (int c = lane; c < C; c += 32) se += expf(z[c] - mx);
+            for (int j = 0; j < kRegs; ++j) {
+                const int c = lane + 32 * j;
+                v[j] = c < C ? z[c] : -INFINITY;
+                mx = fmaxf(mx, v[j]);
+            }
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
-        const float inv_se = 1.0f / se;
-        for (int c = lane; c < C; c += 32) {
-            float g = expf(z[c] - mx) * inv_se;
-            if (c == y) g -= 1.0f;
-            dZ[row * ldz + c] = __float2bfloat16_rn(bad ? NAN : g * invB);
+            for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+#pragma unroll
+            for (int j = 0; j < kRegs; ++j) {
+                v[j] = lane + 32 * j < C ? expf(v[j] - mx) : 0.f;
+                se += v[j];
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
+            const float inv_se = 1.0f / se;
+#pragma unroll
+            for (int j = 0; j < kRegs; ++j) {
+                const int c = lane + 32 * j;
+                if (c < C) {
+                    float g = v[j] * inv_se;
+                    if (c == y) g -= 1.0f;
+                    dZ[row * ldz + c] = __float2bfloat16_rn(bad ? NAN : g * invB);
+                }
+            }
+        } else {
+            for (int c = lane; c < C; c += 32) mx = fmaxf(mx, z[c]);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            for (int c = lane; c < C; c += 32) se += expf(z[c] - mx);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
+            const float inv_se = 1.0f / se;
+            for (int c = lane; c < C; c += 32) {
+                float g = expf(z[c] - mx) * inv_se;
+                if (c == y) g -= 1.0f;
+                dZ[row * ldz + c] = __float2bfloat16_rn(bad ? NAN : g * invB);
+            }
         }
         if (lane == 0) {
             sample_loss[row] = bad ? NAN : (mx + logf(se)) - z[y];
@@ -358,10 +388,12 @@ struct FinishArgs {
 //   vals[n] = sum_j ||g_j||^2 - k ||g_t||^2, the deviation sum of Eq. (10) by the
 //             identity sum_j ||g_j - g_t||^2 = sum_j ||g_j||^2 - k ||g_t||^2 (fp64).
 // Every sum runs in a fixed order (strided per thread, then a fixed tree).
-__global__ void __launch_bounds__(256) finish_received_kernel(FinishArgs a, const int32_t* __restrict__ sel,
-                                                              const int* __restrict__ kdev,
-                                                              double* __restrict__ partials) {
-    __shared__ double red[2][256];
+constexpr int kFinishThreads = 256;
+
+__global__ void __launch_bounds__(kFinishThreads) finish_received_kernel(FinishArgs a, const int32_t* __restrict__ sel,
+                                                                         const int* __restrict__ kdev,
+                                                                         double* __restrict__ partials) {
+    __shared__ double red[2][kFinishThreads];
     const int t = threadIdx.x, n = a.n;
     const int k = *kdev;
     int64_t* hdr = reinterpret_cast<int64_t*>(partials);
@@ -372,15 +404,15 @@ __global__ void __launch_bounds__(256) finish_received_kernel(FinishArgs a, cons
         hdr[2] = n;
         hdr[3] = 0;
     }
-    for (int j = t; j < n; j += 256) vals[j] = 0.0;
+    for (int j = t; j < n; j += kFinishThreads) vals[j] = 0.0;
     double g2 = 0.0, rs = 0.0;
     for (int l = 0; l < a.L; ++l) {
-        for (int64_t i = t; i < a.npw[l]; i += 256) g2 += a.pw[l][i];
-        for (int i = t; i < a.npb[l]; i += 256) g2 += a.pb[l][i];
+        for (int64_t i = t; i < a.npw[l]; i += kFinishThreads) g2 += a.pw[l][i];
+        for (int i = t; i < a.npb[l]; i += kFinishThreads) g2 += a.pb[l][i];
     }
     __syncthreads();   // zeros above land before the received rows below
     const int groups = a.B / 32;   // 32-row groups per worker
-    for (int s = t; s < k; s += 256) {
+    for (int s = t; s < k; s += kFinishThreads) {
         double v = 0.0;
         for (int l = 0; l < a.L; ++l) {
             const double* pg = a.pg[l] + static_cast<int64_t>(s) * groups * a.CT;
@@ -392,7 +424,7 @@ __global__ void __launch_bounds__(256) finish_received_kernel(FinishArgs a, cons
     red[0][t] = g2;
     red[1][t] = rs;
     __syncthreads();
-    for (int h = 128; h > 0; h >>= 1) {
+    for (int h = kFinishThreads / 2; h > 0; h >>= 1) {
         if (t < h) {
             red[0][t] += red[0][t + h];
             red[1][t] += red[1][t + h];
@@ -719,7 +751,7 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
         fa.npb[l] = P.npb[l];
         fa.pg[l] = f64(P.off_pg[l]);
     }
-    finish_received_kernel<<<1, 256, 0, st>>>(fa, sel, kdev, partials);
+    finish_received_kernel<<<1, kFinishThreads, 0, st>>>(fa, sel, kdev, partials);
     e = cudaGetLastError();
     if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
     return DBW_OK;
