@@ -41,6 +41,8 @@ RX_B256 = _wl("rx_b256", (200, 64, 12), 3, 256, 94)
 # k B long enough for the mean-gradient GEMM to split K over several work items (its
 # outputs have far fewer tiles than SMs); b = 31 leaves one worker, so most splits are empty
 RX_SPLIT = _wl("rx_split", (256, 96, 10), 32, 64, 96)
+# a single worker (n = 1): one 32-row slot, k = 1
+RX_ONE = _wl("rx_one", (512, 384, 10), 1, 32, 98)
 
 
 def slot_rows(mask, B):
@@ -109,7 +111,8 @@ def check_against_oracle(it, wl, w0, idx, times, b, workers=None):
 
 
 @pytest.mark.parametrize("wl,b", [(RX_B32, 0), (RX_B32, 3), (RX_B32, 7), (RX_B64, 0), (RX_B64, 2),
-                                  (RX_B128, 1), (RX_B256, 0), (RX_B256, 2), (RX_SPLIT, 5), (RX_SPLIT, 31)],
+                                  (RX_B128, 1), (RX_B256, 0), (RX_B256, 2), (RX_SPLIT, 5), (RX_SPLIT, 31),
+                                  (RX_ONE, 0)],
                          ids=lambda v: v.key if hasattr(v, "key") else f"b{v}")
 def test_received_iteration_matches_oracle(wl, b):
     """All outputs of one received-workers iteration against the oracle: loss (NaN for
