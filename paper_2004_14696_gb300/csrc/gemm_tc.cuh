@@ -75,21 +75,21 @@ struct TcOperands {
 int tc_gemm_mean_dx(const TcOperands& g, const TcEpi& ge, const TcOperands& x, const TcEpi& xe, int* status,
                     cudaStream_t st);
 
-// Per-worker squared gradient norms of one layer without forming the gradient
-// (the Gram identity ||D^T A||_F^2 = <D D^T, A A^T>_F, with the bias term
-// ||1^T D||^2 = sum of D D^T added):
-//   pieces[(r / 32) * CT + ct] = sum over rows r..r+31 of the 32-row group and the
+// Per-worker squared gradient norms of L layers without forming the gradients, in one
+// launch (the Gram identity ||D^T A||_F^2 = <D D^T, A A^T>_F, with the bias term
+// ||1^T D||^2 = sum of D D^T added), for each layer l:
+//   pieces[l][(r / 32) * CT + ct] = sum over rows r..r+31 of the 32-row group and the
 //   columns c of the same worker (in column tile ct, CT = max(1, B / 128)) of
 //   (D D^T)[r, c] * ((A A^T)[r, c] + 1)
-// for the row groups of the first (*kdev) * B rows.  A = act [rows, ldA] (K = colsA),
-// D = dz [rows, ldD] (K = colsD), both bf16 row-major; B % 32 == 0 and either
-// 128 % B == 0 or B % 128 == 0.  part: tc_gram_partial_floats(rows, B) floats of
-// scratch for the partial products of the K ranges; cnt: tc_gram_items(rows, B)
+// for the row groups of the first (*kdev) * B rows.  A = act[l] [rows, ldA[l]] (K =
+// colsA[l]), D = dz[l] [rows, ldD] (K = colsD[l]), both bf16 row-major; B % 32 == 0 and
+// either 128 % B == 0 or B % 128 == 0.  part: tc_gram_partial_floats(rows, B, L) floats
+// of scratch for the partial products of the K ranges; cnt: tc_gram_items(rows, B, L)
 // int32 counters, zero on entry and left zero on return.
-int tc_gram(const __nv_bfloat16* act, int64_t ldA, int64_t colsA, const __nv_bfloat16* dz, int64_t ldD,
-            int64_t colsD, int rows, int B, const int* kdev, double* pieces, float* part, int* cnt, int* status,
-            cudaStream_t st);
-size_t tc_gram_partial_floats(int rows, int B);
-size_t tc_gram_items(int rows, int B);
+int tc_gram(int L, const __nv_bfloat16* const* act, const int64_t* ldA, const int* colsA,
+            const __nv_bfloat16* const* dz, int64_t ldD, const int* colsD, int rows, int B, const int* kdev,
+            double* const* pieces, float* part, int* cnt, int* status, cudaStream_t st);
+size_t tc_gram_partial_floats(int rows, int B, int L);
+size_t tc_gram_items(int rows, int B, int L);
 
 }  // namespace dbw

@@ -59,7 +59,8 @@ struct RxPlan {
     int CT;                            // Gram column tiles per 128-row tile: max(1, B / 128)
     size_t off_sel;                    // int32 [n]: received workers, increasing
     size_t off_k;                      // int32: k
-    size_t off_bpart;                  // fp32 [ceil(M / 256), max out]: bias column sums per 256-row chunk
+    size_t off_bpart[DBW_LMAX];        // fp32 [ceil(M / 256), out_l]: bias column sums per 256-row chunk
+    size_t off_dzl[DBW_LMAX];          // bf16 [M, ldz]: dZ_l of every layer (the last two in off_dz)
     size_t off_pw[DBW_LMAX];           // fp64 [tiles_l * 8]: pieces of ||g_t(W_l)||^2
     int64_t npw[DBW_LMAX];
     size_t off_pb[DBW_LMAX];           // fp64 [ceil(out_l / 256)]: pieces of ||g_t(b_l)||^2

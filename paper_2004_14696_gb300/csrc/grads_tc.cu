@@ -303,20 +303,43 @@ __global__ void __launch_bounds__(1024) compact_received_kernel(const uint8_t* _
     }
 }
 
-// Bias part of Eqs. (3)-(4), g[o] = (1/k) sum_{r < k B} dZ[r, o], in two steps.
-// bias_rows_kernel: one CTA per (256 columns, 256-row chunk); thread (warp y, lane)
-// sums 8 columns (16-byte loads) over rows y, y + 8, ... of the chunk, and the 8
+// Bias part of Eqs. (3)-(4), g[o] = (1/k) sum_{r < k B} dZ[r, o], for every layer,
+// in two launches.  The layers' blocks sit side by side in x; a block finds its
+// layer in the prefix table cb0 (blocks of 256 columns).
+struct BiasLayers {
+    int L;
+    const __nv_bfloat16* dz[DBW_LMAX];   // dZ_l [M, ldz]
+    int64_t ldz;
+    int out[DBW_LMAX];
+    int cb0[DBW_LMAX + 1];               // first column block of layer l; cb0[L] = all blocks
+    float* part[DBW_LMAX];               // [chunks, out_l] column sums per 256-row chunk
+    float* wb[DBW_LMAX];                 // b_l inside w
+    float* gb[DBW_LMAX];                 // b_l inside g_t (nullable)
+    double* pieces[DBW_LMAX];            // [column blocks of layer l]: pieces of ||g_t(b_l)||^2
+};
+
+__device__ __forceinline__ int bias_layer(const BiasLayers& a, int blk) {
+    int l = 0;
+    while (l + 1 < a.L && blk >= a.cb0[l + 1]) ++l;
+    return l;
+}
+
+// bias_rows_kernel: one CTA per (layer, 256 columns, 256-row chunk); thread (warp y,
+// lane) sums 8 columns (16-byte loads) over rows y, y + 8, ... of the chunk, and the 8
 // warps' sums are added in warp order into part[chunk][o].  Chunks past k B write
 // nothing.
-__global__ void __launch_bounds__(256) bias_rows_kernel(const __nv_bfloat16* __restrict__ dZ, int64_t ldz, int out,
-                                                        int B, const int* __restrict__ kdev, float* __restrict__ part) {
+__global__ void __launch_bounds__(256) bias_rows_kernel(BiasLayers a, int B, const int* __restrict__ kdev) {
     __shared__ float red[8][256];
     const int k = *kdev;
     const int rows = k > 0 ? k * B : 0;
     const int r0 = blockIdx.y * 256;
     if (r0 >= rows) return;
+    const int l = bias_layer(a, blockIdx.x);
+    const int cb = blockIdx.x - a.cb0[l], out = a.out[l];
+    const __nv_bfloat16* dZ = a.dz[l];
+    const int64_t ldz = a.ldz;
     const int lane = threadIdx.x & 31, y = threadIdx.x >> 5;
-    const int c = blockIdx.x * 256 + 8 * lane;
+    const int c = cb * 256 + 8 * lane;
     float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
     const int rend = r0 + 256 < rows ? r0 + 256 : rows;
     if (c + 7 < out) {
@@ -334,32 +357,32 @@ __global__ void __launch_bounds__(256) bias_rows_kernel(const __nv_bfloat16* __r
 #pragma unroll
     for (int j = 0; j < 8; ++j) red[y][8 * lane + j] = acc[j];
     __syncthreads();
-    const int o = blockIdx.x * 256 + threadIdx.x;
+    const int o = cb * 256 + threadIdx.x;
     if (o < out) {
         float t = 0.f;
         for (int q = 0; q < 8; ++q) t += red[q][threadIdx.x];
-        part[static_cast<int64_t>(blockIdx.y) * out + o] = t;
+        a.part[l][static_cast<int64_t>(blockIdx.y) * out + o] = t;
     }
 }
 
-// bias_mean_update_kernel: g[o] = (1/k) sum of the chunks' sums (chunk order),
-// wb[o] -= lr g, gb[o] = g (nullable); the CTA's sum of g^2 (fp64, fixed tree) into
-// pieces[blockIdx.x].
-__global__ void __launch_bounds__(256) bias_mean_update_kernel(const float* __restrict__ part, int out, int B,
-                                                               const int* __restrict__ kdev, float lr,
-                                                               float* __restrict__ wb, float* __restrict__ gb,
-                                                               double* __restrict__ pieces) {
+// bias_mean_update_kernel: one CTA per (layer, 256 columns): g[o] = (1/k) sum of the
+// chunks' sums (chunk order), wb[o] -= lr g, gb[o] = g (nullable); the CTA's sum of g^2
+// (fp64, fixed tree) into pieces[column block].
+__global__ void __launch_bounds__(256) bias_mean_update_kernel(BiasLayers a, int B, const int* __restrict__ kdev,
+                                                               float lr) {
     __shared__ double red[8];
     const int k = *kdev;
     const int chunks = k > 0 ? (k * B + 255) / 256 : 0;
-    const int o = blockIdx.x * 256 + threadIdx.x;
+    const int l = bias_layer(a, blockIdx.x);
+    const int cb = blockIdx.x - a.cb0[l], out = a.out[l];
+    const int o = cb * 256 + threadIdx.x;
     double sq = 0.0;
     if (o < out && k > 0) {
         float t = 0.f;
-        for (int q = 0; q < chunks; ++q) t += part[static_cast<int64_t>(q) * out + o];
+        for (int q = 0; q < chunks; ++q) t += a.part[l][static_cast<int64_t>(q) * out + o];
         const float g = t * (1.0f / static_cast<float>(k));
-        wb[o] = fmaf(-lr, g, wb[o]);
-        if (gb) gb[o] = g;
+        a.wb[l][o] = fmaf(-lr, g, a.wb[l][o]);
+        if (a.gb[l]) a.gb[l][o] = g;
         sq = static_cast<double>(g) * g;
     }
     for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
@@ -368,7 +391,7 @@ __global__ void __launch_bounds__(256) bias_mean_update_kernel(const float* __re
     if (threadIdx.x == 0) {
         double t = 0.0;
         for (int w = 0; w < 8; ++w) t += red[w];
-        pieces[blockIdx.x] = t;
+        a.pieces[l][cb] = t;
     }
 }
 
@@ -602,7 +625,14 @@ bool make_rx_plan(int L, const int32_t* widths, int n, int B, RxPlan* P) {
     P->off_k = take(4);
     int maxout = 0;
     for (int l = 0; l < L; ++l) maxout = g.widths[l + 1] > maxout ? g.widths[l + 1] : maxout;
-    P->off_bpart = take(static_cast<size_t>((g.M + 255) / 256) * maxout * 4);
+    for (int l = 0; l < L; ++l)   // bias column sums per 256-row chunk, per layer
+        P->off_bpart[l] = take(static_cast<size_t>((g.M + 255) / 256) * g.widths[l + 1] * 4);
+    // dZ_l of every layer stays until the bias sums and the Gram norms of all layers run
+    // after the backward pass: the two ping-pong buffers hold the last two layers'
+    for (int l = 0; l < L; ++l) {
+        const int back = L - 1 - l;
+        P->off_dzl[l] = back < 2 ? P->t.off_dz[back] : take(static_cast<size_t>(g.M) * P->t.ldz * 2);
+    }
     for (int l = 0; l < L; ++l) {
         const int fin = g.widths[l], fout = g.widths[l + 1];
         P->npw[l] = static_cast<int64_t>((fout + 127) / 128) * ((fin + 255) / 256) * 8;
@@ -612,8 +642,8 @@ bool make_rx_plan(int L, const int32_t* widths, int n, int B, RxPlan* P) {
         P->off_pg[l] = take(static_cast<size_t>(g.M / 32) * P->CT * 8);
     }
     P->off_dzT2 = take(static_cast<size_t>(maxout > g.widths[0] ? maxout : g.widths[0]) * P->t.M8 * 2);
-    P->off_gpart = take(tc_gram_partial_floats(g.M, B) * 4);
-    P->ngcnt = static_cast<int>(tc_gram_items(g.M, B));
+    P->off_gpart = take(tc_gram_partial_floats(g.M, B, L) * 4);
+    P->ngcnt = static_cast<int>(tc_gram_items(g.M, B, L));
     P->off_gcnt = take(static_cast<size_t>(P->ngcnt) * 4);
     P->ws_bytes = cur;
     return true;
@@ -628,7 +658,6 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
     int* status = reinterpret_cast<int*>(ws + T.off_status);
     int32_t* sel = reinterpret_cast<int32_t*>(ws + P.off_sel);
     int* kdev = reinterpret_cast<int*>(ws + P.off_k);
-    float* bpart = reinterpret_cast<float*>(ws + P.off_bpart);
     auto bf = [&](size_t off) { return reinterpret_cast<__nv_bfloat16*>(ws + off); };
     auto f64 = [&](size_t off) { return reinterpret_cast<double*>(ws + off); };
     const char* what = "dbw_received_grads_update";
@@ -679,20 +708,20 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
     }
     const int C = g.widths[L];
     float* sloss = reinterpret_cast<float*>(ws + T.off_sloss);
-    int cur = 0;
-    softmax_xent_ld_kernel<<<n, 256, 0, st>>>(logits, T.ldlog, C, B, idx, S, labels, sloss, bf(T.off_dz[0]), T.ldz,
-                                              loss, sel, kdev);
+    softmax_xent_ld_kernel<<<n, 256, 0, st>>>(logits, T.ldlog, C, B, idx, S, labels, sloss, bf(P.off_dzl[L - 1]),
+                                              T.ldz, loss, sel, kdev);
     {
         dim3 tg((C + 31) / 32, (M + 31) / 32);
-        transpose_bf16_kernel<<<tg, dim3(32, 8), 0, st>>>(bf(T.off_dz[0]), M, C, T.ldz, bf(T.off_dzT), T.M8, kdev,
+        transpose_bf16_kernel<<<tg, dim3(32, 8), 0, st>>>(bf(P.off_dzl[L - 1]), M, C, T.ldz, bf(T.off_dzT), T.M8, kdev,
                                                           B);
     }
     e = cudaGetLastError();
     if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
 
-    // backward: mean gradient + SGD step and dZ of the layer below (one launch), bias,
-    // Gram norms.  dZ_l^T alternates between two buffers: the dX GEMM writes dZ_{l-1}^T
-    // into one while the mean-gradient GEMM reads dZ_l^T from the other.
+    // backward: per layer the mean gradient with the SGD step and dZ of the layer below in
+    // one launch.  dZ_l^T alternates between two buffers: the dX GEMM writes dZ_{l-1}^T
+    // into one while the mean-gradient GEMM reads dZ_l^T from the other.  dZ_l itself
+    // (row-major) is kept for every layer.
     __nv_bfloat16* dzT[2] = {bf(T.off_dzT), bf(P.off_dzT2)};
     int curT = 0;
     for (int l = L - 1; l >= 0; --l) {
@@ -712,32 +741,58 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
             TcEpi ex{};
             ex.act = bf(T.off_act[l]);
             ex.ldact = T.ldact[l];
-            ex.out = bf(T.off_dz[cur ^ 1]);
+            ex.out = bf(P.off_dzl[l - 1]);
             ex.ldo = T.ldz;
             ex.outT = dzT[curT ^ 1];
             ex.ldT = T.M8;
             ex.kdev = kdev;
             ex.kmul = B;
-            const TcOperands xo{bf(T.off_dz[cur]), T.ldz, M, fout, bf(T.off_wt[l]), T.ldwt[l], fin, fout, M, fin, fout};
+            const TcOperands xo{bf(P.off_dzl[l]), T.ldz, M, fout, bf(T.off_wt[l]), T.ldwt[l], fin, fout, M, fin, fout};
             rc = tc_gemm_mean_dx(go, gb, xo, ex, status, st);
         } else {
             rc = tc_gemm(TC_GBAR, go.A, go.lda, go.rowsA, go.colsA, go.B, go.ldb, go.rowsB, go.colsB, go.M, go.N, go.K,
                          1, 0, gb, status, st);
         }
         if (rc) return rc;
-        bias_rows_kernel<<<dim3((fout + 255) / 256, (M + 255) / 256), 256, 0, st>>>(bf(T.off_dz[cur]), T.ldz, fout,
-                                                                                   B, kdev, bpart);
-        bias_mean_update_kernel<<<P.npb[l], 256, 0, st>>>(bpart, fout, B, kdev, lr, w + g.offb[l],
-                                                           gbar ? gbar + g.offb[l] : nullptr, f64(P.off_pb[l]));
+        curT ^= 1;
+    }
+    // bias part of g_t and its step, every layer in two launches
+    {
+        BiasLayers bl{};
+        bl.L = L;
+        bl.ldz = T.ldz;
+        bl.cb0[0] = 0;
+        for (int l = 0; l < L; ++l) {
+            bl.dz[l] = bf(P.off_dzl[l]);
+            bl.out[l] = g.widths[l + 1];
+            bl.cb0[l + 1] = bl.cb0[l] + P.npb[l];
+            bl.part[l] = reinterpret_cast<float*>(ws + P.off_bpart[l]);
+            bl.wb[l] = w + g.offb[l];
+            bl.gb[l] = gbar ? gbar + g.offb[l] : nullptr;
+            bl.pieces[l] = f64(P.off_pb[l]);
+        }
+        bias_rows_kernel<<<dim3(bl.cb0[L], (M + 255) / 256), 256, 0, st>>>(bl, B, kdev);
+        bias_mean_update_kernel<<<bl.cb0[L], 256, 0, st>>>(bl, B, kdev, lr);
         e = cudaGetLastError();
         if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
-        rc = tc_gram(bf(T.off_act[l]), T.ldact[l], fin, bf(T.off_dz[cur]), T.ldz, fout, M, B, kdev, f64(P.off_pg[l]),
-                     gpart, gcnt, status, st);
-        if (rc) return rc;
-        if (l > 0) {
-            cur ^= 1;
-            curT ^= 1;
+    }
+    // per-worker norms of every layer in one launch
+    {
+        const __nv_bfloat16* acts[DBW_LMAX];
+        const __nv_bfloat16* dzs[DBW_LMAX];
+        int64_t lds[DBW_LMAX];
+        int cin[DBW_LMAX], cout[DBW_LMAX];
+        double* pg[DBW_LMAX];
+        for (int l = 0; l < L; ++l) {
+            acts[l] = bf(T.off_act[l]);
+            lds[l] = T.ldact[l];
+            cin[l] = g.widths[l];
+            dzs[l] = bf(P.off_dzl[l]);
+            cout[l] = g.widths[l + 1];
+            pg[l] = f64(P.off_pg[l]);
         }
+        const int rc = tc_gram(L, acts, lds, cin, dzs, T.ldz, cout, M, B, kdev, pg, gpart, gcnt, status, st);
+        if (rc) return rc;
     }
     FinishArgs fa{};
     fa.L = L;

@@ -9,14 +9,15 @@
 // which reads the B (in + out) inputs of the worker instead of the in x out
 // gradient (the per-example-norm trick, applied per worker).
 //
-// Work item = one 128 x 128 Gram tile of one layer: rows m0 .. m0+127 of the
-// stacked received rows against rows n0 .. n0+127 of the same worker block (the
+// One launch covers every layer.  Work item = one 128 x 128 Gram tile of one layer:
+// rows m0 .. m0+127 of the stacked received rows against rows n0 .. n0+127 of the
+// same worker block (the
 // diagonal tile when B <= 128, so both operands are the same staged tile).  The
 // K blocks of A (K = the layer's input width) followed by those of D (K = its
 // output width) are split into S contiguous ranges, one CTA per (item, range),
-// S chosen on the device from k: for B < 128, as many ranges as the live items
-// leave SMs idle (at most 8); S = 1 when the live items alone fill the SMs or
-// B >= 128.  A CTA's TMA producer streams its range through a ring of stages; the MMA
+// S chosen on the device from k: for B < 128, as many ranges as the live items of
+// all layers leave SMs idle (at most 8); S = 1 when the live items alone fill the
+// SMs or B >= 128.  A CTA's TMA producer streams its range through a ring of stages; the MMA
 // issuer accumulates its part of A A^T into TMEM columns 0..127 and of D D^T into
 // 128..255; the four epilogue warps (one per TMEM lane quarter = 32 rows) write
 // the worker-block columns of both partial products to the workspace (with one
@@ -45,18 +46,31 @@ constexpr int GTHREADS = 192;                   // TMA warp, MMA warp, 4 epilogu
 constexpr int GTILE = GBM * GBK * 2;            // 16 KB per operand tile
 constexpr int GSMAX = 8;                        // most K ranges per item
 
+// The layers of one launch: layer l's operands, widths and pieces.
+struct GramLayers {
+    CUtensorMap tmA[DBW_LMAX], tmD[DBW_LMAX];
+    int colsA[DBW_LMAX], colsD[DBW_LMAX];
+    double* pieces[DBW_LMAX];
+    int L;
+    int items;          // work items per layer: 128-row tiles x CT
+};
+
 __global__ void __launch_bounds__(GTHREADS, 1)
-    tc_gram_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmD, int colsA,
-                   int colsD, int B, int CT, int target_ctas, const int* __restrict__ kdev,
-                   double* __restrict__ pieces, float* __restrict__ part, int* __restrict__ cnt, int* status) {
+    tc_gram_kernel(const __grid_constant__ GramLayers G, int B, int CT, int target_ctas, const int* __restrict__ kdev,
+                   float* __restrict__ part, int* __restrict__ cnt, int* status) {
     const int k = *kdev;
     const long long live = static_cast<long long>(k > 0 ? k : 0) * B;   // received rows
-    const int item = blockIdx.x / GSMAX, s_id = blockIdx.x % GSMAX;
-    const int mb = item / CT, ct = item % CT;
+    const int item = blockIdx.x / GSMAX, s_id = blockIdx.x % GSMAX;    // item over all layers
+    const int layer = item / G.items, litem = item % G.items;
+    const int mb = litem / CT, ct = litem % CT;
     const int m0 = mb * GBM;
     if (m0 >= live) return;                     // whole CTA: no barrier or TMEM touched yet
+    const CUtensorMap& tmA = G.tmA[layer];
+    const CUtensorMap& tmD = G.tmD[layer];
+    double* __restrict__ pieces = G.pieces[layer];
+    const int colsA = G.colsA[layer], colsD = G.colsD[layer];
     const int nk1 = (colsA + GBK - 1) / GBK, nk = nk1 + (colsD + GBK - 1) / GBK;
-    const long long live_items = (live + GBM - 1) / GBM * CT;
+    const long long live_items = (live + GBM - 1) / GBM * CT * G.L;   // over all layers of the launch
     // ranges only for worker blocks narrower than a tile: a 128-column block's
     // partials cost as much traffic as the split saves
     int S = B < GBM ? static_cast<int>(target_ctas / live_items) : 1;
@@ -260,16 +274,26 @@ __global__ void __launch_bounds__(GTHREADS, 1)
 
 }  // namespace
 
-int tc_gram(const __nv_bfloat16* act, int64_t ldA, int64_t colsA, const __nv_bfloat16* dz, int64_t ldD, int64_t colsD,
-            int rows, int B, const int* kdev, double* pieces, float* part, int* cnt, int* status, cudaStream_t st) {
+int tc_gram(int L, const __nv_bfloat16* const* act, const int64_t* ldA, const int* colsA,
+            const __nv_bfloat16* const* dz, int64_t ldD, const int* colsD, int rows, int B, const int* kdev,
+            double* const* pieces, float* part, int* cnt, int* status, cudaStream_t st) {
+    if (L < 1 || L > DBW_LMAX) return fail(DBW_EINVAL, "tc_gram: %d layers", L);
     if (B < 32 || B % 32 || (GBM % B && B % GBM)) return fail(DBW_EUNSUPPORTED, "tc_gram: unsupported B = %d", B);
-    if ((ldA % 8) || (ldD % 8) || (reinterpret_cast<uintptr_t>(act) & 15u) || (reinterpret_cast<uintptr_t>(dz) & 15u))
-        return fail(DBW_EALIGN, "tc_gram: unsupported operand alignment");
-    CUtensorMap ta, td;
-    if (!tc_make_map(&ta, act, rows, colsA, ldA, GBK, GBM) || !tc_make_map(&td, dz, rows, colsD, ldD, GBK, GBM))
-        return fail(DBW_ECUDA, "tc_gram: cuTensorMapEncodeTiled failed");
+    GramLayers G{};
+    G.L = L;
     const int CT = B > GBM ? B / GBM : 1;
-    const int items = (rows + GBM - 1) / GBM * CT;
+    G.items = (rows + GBM - 1) / GBM * CT;
+    for (int l = 0; l < L; ++l) {
+        if ((ldA[l] % 8) || (ldD % 8) || (reinterpret_cast<uintptr_t>(act[l]) & 15u) ||
+            (reinterpret_cast<uintptr_t>(dz[l]) & 15u))
+            return fail(DBW_EALIGN, "tc_gram: unsupported operand alignment");
+        if (!tc_make_map(&G.tmA[l], act[l], rows, colsA[l], ldA[l], GBK, GBM) ||
+            !tc_make_map(&G.tmD[l], dz[l], rows, colsD[l], ldD, GBK, GBM))
+            return fail(DBW_ECUDA, "tc_gram: cuTensorMapEncodeTiled failed");
+        G.colsA[l] = colsA[l];
+        G.colsD[l] = colsD[l];
+        G.pieces[l] = pieces[l];
+    }
     // one or two operand rings; at least 80 KB so that at most two CTAs (2 x 256 TMEM
     // columns) share an SM
     const int ring = (B <= GBM ? 1 : 2) * GSTAGES * GTILE;
@@ -277,23 +301,22 @@ int tc_gram(const __nv_bfloat16* act, int64_t ldA, int64_t colsA, const __nv_bfl
     const int smem = need > 80 * 1024 ? need : 80 * 1024;
     cudaError_t e = cudaFuncSetAttribute(tc_gram_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e == cudaSuccess) {
-        tc_gram_kernel<<<items * GSMAX, GTHREADS, smem, st>>>(ta, td, static_cast<int>(colsA), static_cast<int>(colsD),
-                                                              B, CT, sm_count(), kdev, pieces, part, cnt, status);
+        tc_gram_kernel<<<G.items * L * GSMAX, GTHREADS, smem, st>>>(G, B, CT, sm_count(), kdev, part, cnt, status);
         e = cudaGetLastError();
     }
     if (e != cudaSuccess) return fail(DBW_ECUDA, "tc_gram launch: %s", cudaGetErrorString(e));
     return DBW_OK;
 }
 
-size_t tc_gram_partial_floats(int rows, int B) {
+size_t tc_gram_partial_floats(int rows, int B, int L) {
     const int CT = B > GBM ? B / GBM : 1;
-    const size_t items = static_cast<size_t>((rows + GBM - 1) / GBM) * CT;
+    const size_t items = static_cast<size_t>((rows + GBM - 1) / GBM) * CT * L;
     return items * GSMAX * 2 * GBM * static_cast<size_t>(B <= GBM ? B : GBM);
 }
 
-size_t tc_gram_items(int rows, int B) {
+size_t tc_gram_items(int rows, int B, int L) {
     const int CT = B > GBM ? B / GBM : 1;
-    return static_cast<size_t>((rows + GBM - 1) / GBM) * CT;
+    return static_cast<size_t>((rows + GBM - 1) / GBM) * CT * L;
 }
 
 }  // namespace dbw
