@@ -33,12 +33,10 @@ inline int64_t rup(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 // shared-memory tile, column-major with 8-byte stores along m.  row(m) < 0 makes
 // row m zero.  Used for X (gathered minibatch rows) and for W_l (rows = out).
 template <class RowMap>
-__global__ void __launch_bounds__(256) cast_transpose_tile_kernel(const float* __restrict__ src, int64_t lds,
-                                                                  int rows, int cols, RowMap rowmap,
-                                                                  __nv_bfloat16* __restrict__ out, int64_t ldo,
-                                                                  __nv_bfloat16* __restrict__ outT, int64_t ldT) {
+__device__ __forceinline__ void cast_transpose_tile(const float* __restrict__ src, int64_t lds, int rows, int cols,
+                                                    RowMap rowmap, __nv_bfloat16* __restrict__ out, int64_t ldo,
+                                                    __nv_bfloat16* __restrict__ outT, int64_t ldT, int c0, int m0) {
     __shared__ __nv_bfloat16 tile[64][64 + 8];
-    const int c0 = blockIdx.x * 64, m0 = blockIdx.y * 64;
     const int live = rowmap.live(rows);
     if (m0 >= live) return;
     const int t = threadIdx.x;
@@ -110,11 +108,40 @@ __global__ void __launch_bounds__(256) cast_transpose_tile_kernel(const float* _
     }
 }
 
+template <class RowMap>
+__global__ void __launch_bounds__(256) cast_transpose_tile_kernel(const float* __restrict__ src, int64_t lds,
+                                                                  int rows, int cols, RowMap rowmap,
+                                                                  __nv_bfloat16* __restrict__ out, int64_t ldo,
+                                                                  __nv_bfloat16* __restrict__ outT, int64_t ldT) {
+    cast_transpose_tile(src, lds, rows, cols, rowmap, out, ldo, outT, ldT, blockIdx.x * 64, blockIdx.y * 64);
+}
+
 // Row maps of cast_transpose_tile_kernel.
 struct IdentityRows {   // W_l: row o of the matrix
     __device__ int live(int rows) const { return rows; }
     __device__ int64_t operator()(int m) const { return m; }
 };
+// Every layer's W_l -> bf16 W_l and W_l^T in one launch: the layers' 64 x 64 tiles one
+// after the other in x (t0: first tile of layer l; tx: its tiles per row of tiles).
+struct WeightCasts {
+    int L;
+    const float* w[DBW_LMAX];
+    int fin[DBW_LMAX], fout[DBW_LMAX], tx[DBW_LMAX];
+    int t0[DBW_LMAX + 1];
+    __nv_bfloat16* wb[DBW_LMAX];
+    int64_t ldw[DBW_LMAX];
+    __nv_bfloat16* wt[DBW_LMAX];
+    int64_t ldwt[DBW_LMAX];
+};
+
+__global__ void __launch_bounds__(256) cast_transpose_weights_kernel(WeightCasts a) {
+    int l = 0;
+    while (l + 1 < a.L && static_cast<int>(blockIdx.x) >= a.t0[l + 1]) ++l;
+    const int t = blockIdx.x - a.t0[l];
+    cast_transpose_tile(a.w[l], a.fin[l], a.fout[l], a.fin[l], IdentityRows{}, a.wb[l], a.ldw[l], a.wt[l], a.ldwt[l],
+                        (t % a.tx[l]) * 64, (t / a.tx[l]) * 64);
+}
+
 struct GatherRows {     // X of the per-worker pass: pool row idx[m]; an index outside [0, S) reads row 0
     const int32_t* idx;
     int64_t S;
@@ -469,6 +496,27 @@ __global__ void __launch_bounds__(kFinishThreads) finish_received_kernel(FinishA
 
 bool tc_eligible(int prec, int B) { return prec == DBW_PREC_BF16 && B % 32 == 0; }
 
+// bf16 W_l and W_l^T of every layer (one launch).
+static void launch_weight_casts(const TcPlan& P, const float* w, char* ws, cudaStream_t st) {
+    const GradsPlan& g = P.g;
+    WeightCasts a{};
+    a.L = g.L;
+    a.t0[0] = 0;
+    for (int l = 0; l < g.L; ++l) {
+        const int fin = g.widths[l], fout = g.widths[l + 1];
+        a.w[l] = w + g.offW[l];
+        a.fin[l] = fin;
+        a.fout[l] = fout;
+        a.tx[l] = (fin + 63) / 64;
+        a.t0[l + 1] = a.t0[l] + a.tx[l] * ((fout + 63) / 64);
+        a.wb[l] = reinterpret_cast<__nv_bfloat16*>(ws + P.off_wb[l]);
+        a.ldw[l] = P.ldw[l];
+        a.wt[l] = reinterpret_cast<__nv_bfloat16*>(ws + P.off_wt[l]);
+        a.ldwt[l] = P.ldwt[l];
+    }
+    cast_transpose_weights_kernel<<<a.t0[g.L], 256, 0, st>>>(a);
+}
+
 bool make_tc_plan(int L, const int32_t* widths, int n, int B, TcPlan* P) {
     GradsPlan g;
     if (!make_grads_plan(L, widths, n, B, DBW_PREC_BF16, &g)) return false;
@@ -517,12 +565,7 @@ int worker_grads_tc(const TcPlan& P, const float* w, const float* pool, int64_t 
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_worker_grads: %s", cudaGetErrorString(e));
 
     // bf16 weights and their transposes
-    for (int l = 0; l < L; ++l) {
-        const int fin = g.widths[l], fout = g.widths[l + 1];
-        dim3 grid((fin + 63) / 64, (fout + 63) / 64);
-        cast_transpose_tile_kernel<<<grid, 256, 0, st>>>(w + g.offW[l], fin, fout, fin, IdentityRows{},
-                                                         bf(P.off_wb[l]), P.ldw[l], bf(P.off_wt[l]), P.ldwt[l]);
-    }
+    launch_weight_casts(P, w, ws, st);
     // X and X^T
     {
         const int in = g.widths[0];
@@ -667,12 +710,7 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
     int* gcnt = reinterpret_cast<int*>(ws + P.off_gcnt);
     float* gpart = reinterpret_cast<float*>(ws + P.off_gpart);
     compact_received_kernel<<<1, 1024, 0, st>>>(mask, n, sel, kdev, loss, gcnt, P.ngcnt);
-    for (int l = 0; l < L; ++l) {
-        const int fin = g.widths[l], fout = g.widths[l + 1];
-        dim3 grid((fin + 63) / 64, (fout + 63) / 64);
-        cast_transpose_tile_kernel<<<grid, 256, 0, st>>>(w + g.offW[l], fin, fout, fin, IdentityRows{},
-                                                         bf(T.off_wb[l]), T.ldw[l], bf(T.off_wt[l]), T.ldwt[l]);
-    }
+    launch_weight_casts(T, w, ws, st);
     {
         const int in = g.widths[0];
         dim3 grid((in + 63) / 64, (M + 63) / 64);
