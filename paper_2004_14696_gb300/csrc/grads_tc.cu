@@ -203,6 +203,23 @@ __global__ void transpose_bf16_kernel(const __nv_bfloat16* __restrict__ src, int
 // With ``sel`` (received-workers pass): CTA s handles slot s, i.e. worker sel[s]
 // (stacked rows s B .., samples idx[sel[s] B + r], loss[sel[s]]); slots s >= k
 // zero their dZ rows up to the live row count and stop.
+// With ``dZT`` the CTA also writes its rows of the transposed copy dZT [C, ldT]
+// (columns i B .. i B + B - 1): the bf16 values go through a [B, C + 8] shared tile
+// (dynamic shared memory) and leave as 16-byte pieces of 8 rows.
+__device__ __forceinline__ void write_dzT(const __nv_bfloat16* tile, int C, int B, int64_t col0, int rows_live,
+                                          __nv_bfloat16* __restrict__ dZT, int64_t ldT) {
+    const int groups = B / 8;   // B % 32 == 0 on the tcgen05 path
+    for (int q = threadIdx.x; q < C * groups; q += blockDim.x) {
+        const int c = q / groups, g8 = q % groups;
+        if (8 * g8 >= rows_live) continue;
+        uint4 v;
+        __nv_bfloat16* h = reinterpret_cast<__nv_bfloat16*>(&v);
+#pragma unroll
+        for (int t = 0; t < 8; ++t) h[t] = tile ? tile[(8 * g8 + t) * (C + 8) + c] : __float2bfloat16_rn(0.f);
+        *reinterpret_cast<uint4*>(dZT + static_cast<int64_t>(c) * ldT + col0 + 8 * g8) = v;
+    }
+}
+
 __global__ void __launch_bounds__(256) softmax_xent_ld_kernel(const float* __restrict__ logits, int64_t ldl, int C,
                                                               int B, const int32_t* __restrict__ idx, int64_t S,
                                                               const int32_t* __restrict__ labels,
@@ -210,7 +227,10 @@ __global__ void __launch_bounds__(256) softmax_xent_ld_kernel(const float* __res
                                                               __nv_bfloat16* __restrict__ dZ, int64_t ldz,
                                                               float* __restrict__ loss,
                                                               const int32_t* __restrict__ sel = nullptr,
-                                                              const int* __restrict__ kdev = nullptr) {
+                                                              const int* __restrict__ kdev = nullptr,
+                                                              __nv_bfloat16* __restrict__ dZT = nullptr,
+                                                              int64_t ldT = 0) {
+    extern __shared__ __nv_bfloat16 tileT[];   // [B][C + 8] when dZT is given
     const int i = blockIdx.x;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
     int worker = i;
@@ -220,6 +240,7 @@ __global__ void __launch_bounds__(256) softmax_xent_ld_kernel(const float* __res
             for (int r = warp; r < B && i * B + r < live; r += nw)
                 for (int c = lane; c < C; c += 32)
                     dZ[(static_cast<int64_t>(i) * B + r) * ldz + c] = __float2bfloat16_rn(0.f);
+            if (dZT) write_dzT(nullptr, C, B, static_cast<int64_t>(i) * B, live - i * B, dZT, ldT);
             return;
         }
         worker = sel[i];
@@ -262,7 +283,9 @@ __global__ void __launch_bounds__(256) softmax_xent_ld_kernel(const float* __res
                 if (c < C) {
                     float g = v[j] * inv_se;
                     if (c == y) g -= 1.0f;
-                    dZ[row * ldz + c] = __float2bfloat16_rn(bad ? NAN : g * invB);
+                    const __nv_bfloat16 h = __float2bfloat16_rn(bad ? NAN : g * invB);
+                    dZ[row * ldz + c] = h;
+                    if (dZT) tileT[r * (C + 8) + c] = h;
                 }
             }
         } else {
@@ -276,7 +299,9 @@ __global__ void __launch_bounds__(256) softmax_xent_ld_kernel(const float* __res
             for (int c = lane; c < C; c += 32) {
                 float g = expf(z[c] - mx) * inv_se;
                 if (c == y) g -= 1.0f;
-                dZ[row * ldz + c] = __float2bfloat16_rn(bad ? NAN : g * invB);
+                const __nv_bfloat16 h = __float2bfloat16_rn(bad ? NAN : g * invB);
+                dZ[row * ldz + c] = h;
+                if (dZT) tileT[r * (C + 8) + c] = h;
             }
         }
         if (lane == 0) {
@@ -290,6 +315,14 @@ __global__ void __launch_bounds__(256) softmax_xent_ld_kernel(const float* __res
         for (int r = 0; r < B; ++r) acc += sample_loss[static_cast<int64_t>(i) * B + r];
         loss[worker] = bad_s ? NAN : acc * invB;
     }
+    if (dZT) write_dzT(tileT, C, B, static_cast<int64_t>(i) * B, B, dZT, ldT);
+}
+
+// Shared memory of softmax_xent_ld_kernel's transposing tile, or 0 when it does not
+// fit (the transpose then runs as transpose_bf16_kernel).
+inline int softmax_tile_bytes(int B, int C) {
+    const long long bytes = static_cast<long long>(B) * (C + 8) * 2;
+    return bytes <= 160 * 1024 ? static_cast<int>(bytes) : 0;
 }
 
 // G[i, offb + o] = sum_{r < B} dZ[i*B + r, o] (rows in order).
@@ -602,9 +635,14 @@ int worker_grads_tc(const TcPlan& P, const float* w, const float* pool, int64_t 
     const int C = g.widths[L];
     float* sloss = reinterpret_cast<float*>(ws + P.off_sloss);
     int cur = 0;
-    softmax_xent_ld_kernel<<<n, 256, 0, st>>>(logits, P.ldlog, C, B, idx, S, labels, sloss, bf(P.off_dz[0]), P.ldz,
-                                              loss);
-    {
+    if (const int tb = softmax_tile_bytes(B, C)) {
+        e = cudaFuncSetAttribute(softmax_xent_ld_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, tb);
+        if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_worker_grads: %s", cudaGetErrorString(e));
+        softmax_xent_ld_kernel<<<n, 256, tb, st>>>(logits, P.ldlog, C, B, idx, S, labels, sloss, bf(P.off_dz[0]),
+                                                   P.ldz, loss, nullptr, nullptr, bf(P.off_dzT), P.M8);
+    } else {
+        softmax_xent_ld_kernel<<<n, 256, 0, st>>>(logits, P.ldlog, C, B, idx, S, labels, sloss, bf(P.off_dz[0]),
+                                                  P.ldz, loss);
         dim3 tg((C + 31) / 32, (M + 31) / 32);
         transpose_bf16_kernel<<<tg, dim3(32, 8), 0, st>>>(bf(P.off_dz[0]), M, C, P.ldz, bf(P.off_dzT), P.M8);
     }
@@ -746,9 +784,14 @@ int received_grads_tc(const RxPlan& P, float* w, const float* pool, int64_t S, c
     }
     const int C = g.widths[L];
     float* sloss = reinterpret_cast<float*>(ws + T.off_sloss);
-    softmax_xent_ld_kernel<<<n, 256, 0, st>>>(logits, T.ldlog, C, B, idx, S, labels, sloss, bf(P.off_dzl[L - 1]),
-                                              T.ldz, loss, sel, kdev);
-    {
+    if (const int tb = softmax_tile_bytes(B, C)) {
+        e = cudaFuncSetAttribute(softmax_xent_ld_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, tb);
+        if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+        softmax_xent_ld_kernel<<<n, 256, tb, st>>>(logits, T.ldlog, C, B, idx, S, labels, sloss,
+                                                   bf(P.off_dzl[L - 1]), T.ldz, loss, sel, kdev, bf(T.off_dzT), T.M8);
+    } else {
+        softmax_xent_ld_kernel<<<n, 256, 0, st>>>(logits, T.ldlog, C, B, idx, S, labels, sloss, bf(P.off_dzl[L - 1]),
+                                                  T.ldz, loss, sel, kdev);
         dim3 tg((C + 31) / 32, (M + 31) / 32);
         transpose_bf16_kernel<<<tg, dim3(32, 8), 0, st>>>(bf(P.off_dzl[L - 1]), M, C, T.ldz, bf(T.off_dzT), T.M8, kdev,
                                                           B);

@@ -195,16 +195,18 @@ class Iteration:
         reduce kernel, which this count leaves out."""
         L = len(self.wl.widths) - 1
         choose = (0 if self.static_b is not None else 1) + (3 if self.clock == "psw" else 0)   # + arrivals, record, fit
+        # loss + dZ (+ dZ^T, written by the same kernel when its transposing tile fits)
+        loss = 1 if self.wl.B * (self.wl.widths[-1] + 8) * 2 <= 160 * 1024 else 2
         if self.received:
             # select; compaction, the weight cast-transposes of all layers (1), X and X^T, L forward
             # GEMMs, loss + dZ^T, per layer the mean-gradient GEMM (with the dX GEMM in the same
             # launch when l > 0); bias row sums and bias mean of all layers (2), Gram norms of all
             # layers (1), finish; grad_stats (2)
-            return choose + 1 + (1 + 1 + 1 + L + 2 + L + 2 + 1 + 1) + 2
+            return choose + 1 + (1 + 1 + 1 + L + loss + L + 2 + 1 + 1) + 2
         if self.wl.prec == dbw.PREC_BF16 and self.wl.B % 32 == 0:
             # tcgen05 pass: the weight cast-transposes of all layers (1), X and X^T, L forward GEMMs,
             # loss + dZ^T, L dW GEMMs, L bias gradients, L-1 dX GEMMs
-            grads = 1 + 1 + L + 2 + L + L + (L - 1)
+            grads = 1 + 1 + L + loss + L + L + (L - 1)
         else:
             grads = 1 + L + 1 + L + L + (L - 1)    # gather, forward, loss, dW, bias, dX
             if self.wl.prec == dbw.PREC_BF16:
