@@ -387,9 +387,11 @@ __global__ void __launch_bounds__(kThreads, MINB)
 // two thirds of what the single-CTA tile stages for the same work, so the ring
 // is deeper in the same shared memory and each SM pulls fewer bytes per flop.
 //
-// One launch may carry two independent problems (KIND1 != KIND0 or p[1] live):
-// their tiles form one list, those of problem 0 first, dealt to the pairs in
-// turn, so that the second problem fills the last partial wave of the first.
+// One launch may carry two independent problems (nprob = 2, kinds KIND0 and
+// KIND1): their tiles form one list, those of problem 0 first, dealt to the pairs
+// in turn, so that the second problem fills the last partial wave of the first.
+// Shared memory: the ring of STAGES stages, 256 bytes of barriers, then a 32 x 32
+// bf16 transposing chunk per epilogue warp.
 //
 // Barriers (the same shared-memory offsets in both CTAs):
 //   full[s]    even CTA only: its producer arrives with the byte count of both
