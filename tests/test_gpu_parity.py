@@ -325,6 +325,12 @@ UNALIGNED_BF16 = workloads.Workload(
     key="unaligned_bf16", widths=(36, 18, 10), n=2, B=32, prec=workloads.PREC_BF16, S=200,
     feature_dist="normal", time_model="shifted_exp", time_params={"shift": 1.0, "rate": 1.0}, lr=0.01,
     seed_offset=81)
+# B (C + 8) bf16 larger than the softmax kernel's transposing tile: dZ_L^T by the separate
+# transpose kernel
+WIDE_BF16 = workloads.Workload(
+    key="wide_bf16", widths=(64, 320), n=2, B=256, prec=workloads.PREC_BF16, S=600,
+    feature_dist="normal", time_model="shifted_exp", time_params={"shift": 1.0, "rate": 1.0}, lr=0.01,
+    seed_offset=82)
 SMALL_FP32_RAGGED = workloads.Workload(
     key="small_fp32", widths=(132, 200, 70, 7), n=5, B=3, prec=workloads.PREC_FP32, S=50,
     feature_dist="uniform", time_model="pareto", time_params={"alpha": 2.0, "xm": 1.0}, lr=0.05, seed_offset=78)
@@ -341,7 +347,7 @@ def grads_case(wl, t=0):
 
 
 @pytest.mark.parametrize("wl", [workloads.SOFTMAX784, workloads.MLP784, SMALL_FP32_RAGGED, SMALL_BF16,
-                                SMALL_BF16_SIMT, ODD_BF16, UNALIGNED_BF16], ids=lambda w: w.key)
+                                SMALL_BF16_SIMT, ODD_BF16, UNALIGNED_BF16, WIDE_BF16], ids=lambda w: w.key)
 def test_worker_grads_parity_full(wl):
     it, idx = grads_case(wl)
     pool, labels, w = it.pool.cpu().numpy(), it.labels.cpu().numpy(), it.w.cpu().numpy()

@@ -43,6 +43,9 @@ RX_B256 = _wl("rx_b256", (200, 64, 12), 3, 256, 94)
 RX_SPLIT = _wl("rx_split", (256, 96, 10), 32, 64, 96)
 # a single worker (n = 1): one 32-row slot, k = 1
 RX_ONE = _wl("rx_one", (512, 384, 10), 1, 32, 98)
+# B (C + 8) bf16 larger than the softmax kernel's transposing tile: dZ_L^T by the separate
+# transpose kernel
+RX_WIDE = _wl("rx_wide", (64, 320), 3, 256, 99)
 
 
 def slot_rows(mask, B):
@@ -112,7 +115,7 @@ def check_against_oracle(it, wl, w0, idx, times, b, workers=None):
 
 @pytest.mark.parametrize("wl,b", [(RX_B32, 0), (RX_B32, 3), (RX_B32, 7), (RX_B64, 0), (RX_B64, 2),
                                   (RX_B128, 1), (RX_B256, 0), (RX_B256, 2), (RX_SPLIT, 5), (RX_SPLIT, 31),
-                                  (RX_ONE, 0)],
+                                  (RX_ONE, 0), (RX_WIDE, 1)],
                          ids=lambda v: v.key if hasattr(v, "key") else f"b{v}")
 def test_received_iteration_matches_oracle(wl, b):
     """All outputs of one received-workers iteration against the oracle: loss (NaN for
