@@ -16,8 +16,8 @@
 // K blocks of A (K = the layer's input width) followed by those of D (K = its
 // output width) are split into S contiguous ranges, one CTA per (item, range),
 // S chosen on the device from k: for B < 128, as many ranges as the live items of
-// all layers leave SMs idle (at most 8); S = 1 when the live items alone fill the
-// SMs or B >= 128.  A CTA's TMA producer streams its range through a ring of stages; the MMA
+// all layers leave slots idle at two CTAs per SM (at most 8); S = 1 when the live
+// items alone fill them or B >= 128.  A CTA's TMA producer streams its range through a ring of stages; the MMA
 // issuer accumulates its part of A A^T into TMEM columns 0..127 and of D D^T into
 // 128..255; the four epilogue warps (one per TMEM lane quarter = 32 rows) write
 // the worker-block columns of both partial products to the workspace (with one
@@ -301,7 +301,9 @@ int tc_gram(int L, const __nv_bfloat16* const* act, const int64_t* ldA, const in
     const int smem = need > 80 * 1024 ? need : 80 * 1024;
     cudaError_t e = cudaFuncSetAttribute(tc_gram_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e == cudaSuccess) {
-        tc_gram_kernel<<<G.items * L * GSMAX, GTHREADS, smem, st>>>(G, B, CT, sm_count(), kdev, part, cnt, status);
+        // ranges sized for two resident CTAs per SM
+        tc_gram_kernel<<<G.items * L * GSMAX, GTHREADS, smem, st>>>(G, B, CT, 2 * sm_count(), kdev, part, cnt,
+                                                                     status);
         e = cudaGetLastError();
     }
     if (e != cudaSuccess) return fail(DBW_ECUDA, "tc_gram launch: %s", cudaGetErrorString(e));
