@@ -544,7 +544,8 @@ static void launch_weight_casts(const TcPlan& P, const float* w, char* ws, cudaS
         a.t0[l + 1] = a.t0[l] + a.tx[l] * ((fout + 63) / 64);
         a.wb[l] = reinterpret_cast<__nv_bfloat16*>(ws + P.off_wb[l]);
         a.ldw[l] = P.ldw[l];
-        a.wt[l] = reinterpret_cast<__nv_bfloat16*>(ws + P.off_wt[l]);
+        // no input gradient is formed for the first layer: W_0^T is never read
+        a.wt[l] = l == 0 ? nullptr : reinterpret_cast<__nv_bfloat16*>(ws + P.off_wt[l]);
         a.ldwt[l] = P.ldwt[l];
     }
     cast_transpose_weights_kernel<<<a.t0[g.L], 256, 0, st>>>(a);
