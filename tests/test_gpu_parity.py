@@ -84,6 +84,19 @@ def test_select_bit_exact(n):
             assert int(got["k"][0]) == n - b
 
 
+def test_select_negative_times_and_signed_zeros():
+    """The comparisons order the doubles themselves: negative times, subnormals, and -0
+    equal to +0 (so their tie goes to the lower index), as the oracle's sort does."""
+    times = np.array([0.0, -0.0, -1.5, 2.0, -5e-324, 5e-324, -0.0, 0.0, 3.0, -2.0, -1.5, 1e300, -1e300, 2.0],
+                     dtype=np.float64)
+    for b in range(len(times)):
+        got = gpu_select(times, b)
+        order, mask, ts = O.select_fastest(times, b)
+        assert np.array_equal(got["order"], order)
+        assert np.array_equal(got["mask"], mask)
+        assert same_f64(got["tsorted"], ts)
+
+
 def test_select_clamps_out_of_range_b():
     times = np.random.default_rng(0).exponential(size=10)
     assert int(gpu_select(times, -3)["k"][0]) == 10
