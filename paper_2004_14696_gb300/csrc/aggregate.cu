@@ -10,7 +10,8 @@
 // (128 * VEC columns); a persistent grid of warps walks the chunks.  A warp owns
 // its chunk for all k received rows, so the column reductions stay in its lanes'
 // registers: no shared memory and no block barrier in the streaming loop.  Rows
-// are processed UNROLL at a time to keep several 128-bit loads in flight per lane.
+// are processed UNROLL at a time, and the next batch's 128-bit loads are issued
+// before the current batch is reduced.
 //
 // Numerics.  Per column the warp keeps s1 = sum (x - c) and s2 = sum (x - c)^2 in
 // fp32 with the shift c = the column's value in the first received row, so that
@@ -28,7 +29,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int VEC = 2;      // float4 per lane per row: chunk = 32 * VEC * 4 = 256 columns
-constexpr int UNROLL = 4;   // rows in flight per lane
+constexpr int UNROLL = 2;   // rows per batch; two batches in flight per lane
 constexpr int kChunkCols = 32 * VEC * 4;
 
 __device__ __forceinline__ float4 ldg_stream(const float4* p) {
@@ -123,17 +124,36 @@ __global__ void __launch_bounds__(kThreads, 3) aggregate_kernel(
             rn = warp_sum(rn);
             if (lane == 0) myrow[0] += (double)rn;
         }
+        // rows 1 .. k-1 in batches of UNROLL; the next batch's loads are in flight while
+        // this batch is reduced
+        float4 xn[UNROLL][VEC];
+#pragma unroll
+        for (int u = 0; u < UNROLL; ++u) {
+            const int p = 1 + u;
+            const float* rowp = G + (int64_t)sel[p < k ? p : 0] * ld;
+#pragma unroll
+            for (int v = 0; v < VEC; ++v) {
+                const int64_t col = col0 + v * 128;
+                xn[u][v] = (p < k && inb[v]) ? ldg_stream(reinterpret_cast<const float4*>(rowp + col)) : c[v];
+            }
+        }
         for (int p0 = 1; p0 < k; p0 += UNROLL) {
             float4 x[UNROLL][VEC];
 #pragma unroll
-            for (int u = 0; u < UNROLL; ++u) {
-                const int p = p0 + u;
-                const float* rowp = G + (int64_t)sel[p < k ? p : 0] * ld;
+            for (int u = 0; u < UNROLL; ++u)
 #pragma unroll
-                for (int v = 0; v < VEC; ++v) {
-                    const int64_t col = col0 + v * 128;
-                    x[u][v] = (p < k && inb[v]) ? ldg_stream(reinterpret_cast<const float4*>(rowp + col))
-                                                : c[v];
+                for (int v = 0; v < VEC; ++v) x[u][v] = xn[u][v];
+            if (p0 + UNROLL < k) {
+#pragma unroll
+                for (int u = 0; u < UNROLL; ++u) {
+                    const int p = p0 + UNROLL + u;
+                    const float* rowp = G + (int64_t)sel[p < k ? p : 0] * ld;
+#pragma unroll
+                    for (int v = 0; v < VEC; ++v) {
+                        const int64_t col = col0 + v * 128;
+                        xn[u][v] = (p < k && inb[v]) ? ldg_stream(reinterpret_cast<const float4*>(rowp + col))
+                                                     : c[v];
+                    }
                 }
             }
 #pragma unroll
