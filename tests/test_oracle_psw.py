@@ -374,3 +374,98 @@ def test_more_idle_workers_at_start_is_faster():
         m3 = ps.sums[3, i] / ps.cnts[3, i]
         m6 = ps.sums[6, i] / ps.cnts[6, i]
         assert m6 < m3, (i, m6, m3)
+
+
+# ---------------------------------------------------------------- P3 (b): diagonal cells outside group (a)
+# Hand-worked cell tables: every expected T^_k below is worked out by hand from P3's
+# rule (pooled column means, the nearest sampled column before else after for an
+# empty column, PAVA with unit weights over the cells outside group (a), clipped to
+# the bounds the order of Eq. (17) puts on them), not by the oracle's code.
+def table(n, cells):
+    """A push-and-wait state whose cell (h, i) holds samples summing to s, c of them."""
+    ps = P.psw_init(n)
+    for (h, i), (s, c) in cells.items():
+        ps.sums[h, i] = s
+        ps.cnts[h, i] = c
+    return ps
+
+
+# n = 5.  Group (a) = row 3 alone: cells 1, 2, 3 already increasing, so the fit
+# keeps them.  Row 5 has no diagonal sample.  Column means: col 1 = (1 + 27)/4 = 7,
+# col 2 = (2 + 1)/2 = 1.5, col 4 = 3.5, col 5 empty -> col 4's 3.5.  PAVA over the
+# cells k = 1, 2, 4, 5 of [7, 1.5, 3.5, 3.5]: 7 > 1.5 pools to 4.25 (2 cells), then
+# 4.25 > 3.5 pools to 4 (3 cells), then 4 > 3.5 pools to 3.875 (4 cells).  Bounds
+# from row 3: k = 1: [x31, x33] = [1, 3] -> 3 (clipped from above); k = 2:
+# [x32, x33] = [2, 3] -> 3 (from above); k = 4, 5: [x33, inf) = [3, inf) -> 3.875.
+TABLE_ABOVE = (5, {(3, 1): (1.0, 1), (3, 2): (2.0, 1), (3, 3): (3.0, 1),
+                   (5, 1): (27.0, 3), (5, 2): (1.0, 1), (5, 3): (2.5, 1), (5, 4): (3.5, 1)},
+               [3.0, 3.0, 3.0, 3.875, 3.875])
+# n = 5.  Group (a) = row 2 with the single cell (2, 2), mean 8/2 = 4.  Column 1 is
+# empty with no sampled column before it -> col 2's 4; col 3 = 3; col 4 empty ->
+# col 3's 3 (the column before it, not col 5's 6); col 5 = 6.  PAVA over k = 1, 3, 4, 5
+# of [4, 3, 3, 6]: 4 > 3 pools to 3.5, then 3.5 > 3 pools to 10/3; 6 stays.  Bounds
+# from (2, 2): k = 1: (-inf, 4] -> 10/3; k = 3, 4, 5: [4, inf) -> 4, 4 (clipped from
+# below), 6.
+TABLE_BELOW = (5, {(2, 2): (8.0, 2), (5, 3): (3.0, 1), (4, 5): (6.0, 1)},
+               [10.0 / 3.0, 4.0, 4.0, 4.0, 6.0])
+# n = 4.  Group (a) = rows 2 and 4.  Cells a = (2,1) = 1, b = (2,2) = 4, c = (4,1) = 2,
+# d = (4,2) = 1, e = (4,3) = 3, f = (4,4) = 5.  Eq. (17): a <= b, c <= d <= e <= f
+# (rows), c <= a, d <= b (columns), b <= f (diagonal).  The projection pools
+# {a, c, d} to (1 + 2 + 1)/3 = 4/3: every lower part of that block has a mean >= 4/3
+# ({c} 2, {c, d} 1.5, {c, a} 1.5) and every upper part <= 4/3 ({a} 1, {d} 1), and
+# the result is feasible.  So T^_2 = 4 and T^_4 = 5.  Row 3 has no diagonal sample.
+# Col 1 = (1 + 2 + 0.5)/3 = 7/6, col 3 = 3.  PAVA over k = 1, 3: unchanged.  k = 1:
+# lo = max(x21, x41) = 4/3, hi = min(x22, x44) = 4 -> 4/3 (clipped from below by a
+# pooled value); k = 3: lo = max over row 2 (j <= 2) and row 4 (j <= 3) = 4,
+# hi = x44 = 5 -> 4.
+TABLE_TWO_ROWS = (4, {(2, 1): (1.0, 1), (2, 2): (4.0, 1), (4, 1): (2.0, 1), (4, 2): (1.0, 1), (4, 3): (3.0, 1),
+                      (4, 4): (5.0, 1), (3, 1): (0.5, 1), (3, 2): (6.0, 1)},
+                  [4.0 / 3.0, 4.0, 4.0, 5.0])
+HAND_TABLES = {"clipped_above": TABLE_ABOVE, "clipped_below": TABLE_BELOW, "two_group_rows": TABLE_TWO_ROWS}
+
+
+@pytest.mark.parametrize("name", sorted(HAND_TABLES))
+def test_free_diagonal_cells_hand_worked(name):
+    n, cells, want = HAND_TABLES[name]
+    got = P.time_estimates(table(n, cells))
+    assert np.allclose(got, want, rtol=1e-12, atol=0), (got, want)
+
+
+def test_planted_next_column_fallback_is_caught(monkeypatch):
+    """An empty column that takes the next sampled column's mean instead of the previous one's."""
+    def wrong(ps):
+        n = ps.n
+        col_sum, col_cnt = ps.sums[1:, 1:].sum(axis=0), ps.cnts[1:, 1:].sum(axis=0)
+        mu = np.full(n, math.nan)
+        for i in range(n - 1, -1, -1):
+            if col_cnt[i] > 0:
+                mu[i] = col_sum[i] / col_cnt[i]
+            elif i < n - 1:
+                mu[i] = mu[i + 1]
+        return mu
+    monkeypatch.setattr(P, "column_means", wrong)
+    n, cells, want = TABLE_BELOW
+    assert not np.allclose(P.time_estimates(table(n, cells)), want, rtol=1e-12, atol=0)
+
+
+def test_planted_missing_pava_over_free_cells_is_caught(monkeypatch):
+    """Skipping the PAVA pass (each free cell keeps its own column mean).  Group (a) of
+    this table is one increasing row, which PAVA leaves as it is either way."""
+    monkeypatch.setattr(P, "pava", lambda y, w: np.array(y, dtype=np.float64))
+    n, cells, want = TABLE_ABOVE
+    assert not np.allclose(P.time_estimates(table(n, cells)), want, rtol=1e-12, atol=0)
+
+
+def test_planted_wrong_lower_bound_is_caught(monkeypatch):
+    """A lower bound taken over j <= max(h, k) instead of j <= min(h, k)."""
+    def wrong(fit, k):
+        lo, hi = -math.inf, math.inf
+        for (h, j), xv in fit.items():
+            if j <= max(h, k):
+                lo = max(lo, xv)
+            if j >= max(h, k):
+                hi = min(hi, xv)
+        return lo, hi
+    monkeypatch.setattr(P, "diagonal_bounds", wrong)
+    n, cells, want = TABLE_TWO_ROWS
+    assert not np.allclose(P.time_estimates(table(n, cells)), want, rtol=1e-12, atol=0)
