@@ -224,10 +224,12 @@ int dbw_select_fastest(const double* times, int n, const int32_t* b,
  * Layout of the partials buffer (caller-owned scratch written by
  * dbw_aggregate_update and read by dbw_grad_stats; public so that a caller can
  * also assemble the sums for dbw_grad_stats itself):
- *   int64_t header[4] = {DBW_PARTIALS_MAGIC, blocks, n, 0}
+ *   int64_t header[4] = {DBW_PARTIALS_MAGIC, blocks, n, flags}
+ *           flags: DBW_ALL_ROW_NORMS if every row's norm is in vals, else 0
  *   double  sums[n + 2]              reduced totals, written by dbw_grad_stats
  *   double  vals[(n + 2) * blocks]   per-block pieces, vals[q * blocks + j]:
- *           q < n: piece of ||g_q||^2 (0 for rows not received),
+ *           q < n: piece of ||g_q||^2 (0 for rows not received, unless the
+ *           header carries DBW_ALL_ROW_NORMS),
  *           q = n: piece of the deviation sum of Eq. (10), q = n + 1: piece of ||g_t||^2.
  * dbw_grad_stats reduces each quantity in a fixed order (256 strided fp64
  * partial sums, then a pairwise tree), so equal buffers give equal results.
@@ -247,15 +249,23 @@ size_t dbw_aggregate_partials_bytes(int n, int64_t d);
  * reduces.  Column sums use a per-column shift (the first received row) so that
  * the deviation sum does not cancel; cross-column sums are fp64.
  *
- *  G        [n, ld] fp32, ld % 4 == 0, 16-byte aligned; only received rows read.
- *  mask     [n] uint8 from dbw_select_fastest (at least one byte set).
+ *  G        [n, ld] fp32, ld % 4 == 0, 16-byte aligned; only received rows read
+ *           (every row with DBW_ALL_ROW_NORMS).
+ *  mask     [n] uint8 from dbw_select_fastest (at least one byte set; with none
+ *           set, w is left as it is and every piece is 0).
  *  w        [d] fp32, updated in place (16-byte aligned).
  *  gbar     [d] fp32 out (nullable, 16-byte aligned): g_t.
+ *  flags    0, or DBW_ALL_ROW_NORMS: also read the n - k rows the mask leaves
+ *           out, for their ||g_j||^2 only ((n - k) d * 4 more bytes).  g_t, w and
+ *           the sums of Eq. (10) still come from the received rows alone (Eq. (10)
+ *           sums over the k received gradients); dbw_grad_stats then reports
+ *           every row's norm in row_sqnorm.  Other bits: DBW_EINVAL.
  *  partials scratch of partials_bytes >= dbw_aggregate_partials_bytes(n, d),
  *           256-byte aligned; consumed by the next dbw_grad_stats.
  */
+#define DBW_ALL_ROW_NORMS 1
 int dbw_aggregate_update(const float* G, int64_t ld, int n, int64_t d,
-                         const uint8_t* mask, float lr, float* w, float* gbar,
+                         const uint8_t* mask, float lr, float* w, float* gbar, int flags,
                          double* partials, size_t partials_bytes, void* stream);
 
 /*
@@ -277,16 +287,19 @@ int dbw_aggregate_update(const float* G, int64_t ld, int n, int64_t d,
  * runtime's cudaGetSymbolAddress, with that device current) and caches it; make
  * that first call before any stream capture begins.  All calls on a device
  * share the array: calls whose GPU work overlaps (unordered streams) race and
- * corrupt each other's sums.  Nothing in the array needs to start at zero.
+ * corrupt each other's sums.  Each call clears the array's header on its stream
+ * before the aggregation, so a call whose aggregation did not run yields NaN
+ * sums rather than an earlier call's; nothing else in it needs to start at zero.
  *
- *  G, ld, n, d, mask, lr, w, gbar   as for dbw_aggregate_update.
+ *  G, ld, n, d, mask, lr, w, gbar, flags   as for dbw_aggregate_update.
  *  sums_out  [n + 2] fp64 device out: sums_out[j] = ||g_j||^2 for received rows
- *            (0 otherwise), sums_out[n] = the deviation sum of Eq. (10),
- *            sums_out[n + 1] = ||g_t||^2 -- the totals dbw_grad_stats would form.
+ *            (0 otherwise; every row with DBW_ALL_ROW_NORMS), sums_out[n] = the
+ *            deviation sum of Eq. (10), sums_out[n + 1] = ||g_t||^2 -- the totals
+ *            dbw_grad_stats would form.
  */
 #define DBW_NOALLOC_SCRATCH_BYTES ((size_t)4 << 20)
 int dbw_aggregate_update_noalloc(const float* G, int64_t ld, int n, int64_t d, const uint8_t* mask, float lr,
-                                 float* w, float* gbar, double* sums_out, void* stream);
+                                 float* w, float* gbar, int flags, double* sums_out, void* stream);
 
 /* Workspace bytes dbw_received_grads_update needs for (widths, n, B, prec); 0 if
  * the shape is invalid or the call does not support it. */
@@ -363,7 +376,9 @@ int dbw_state_init(dbw_state* state, int n, int D, void* stream);
  *  tsorted     [n] from dbw_select_fastest.
  *  lr          the learning rate eta used by the update.
  *  stats_out   [DBW_STATS_LEN] fp64 out (nullable), see DBW_STAT_*.
- *  row_sqnorm  [n] fp64 out (nullable): ||g_j||^2 for received rows, NaN otherwise.
+ *  row_sqnorm  [n] fp64 out (nullable): ||g_j||^2 for received rows, NaN for the
+ *              others -- unless the aggregation ran with DBW_ALL_ROW_NORMS, then
+ *              ||g_j||^2 of every row.
  */
 int dbw_grad_stats(const double* partials, int n, const uint8_t* mask,
                    const float* loss, const double* tsorted, double lr,
@@ -415,7 +430,13 @@ int dbw_choose_b(dbw_state* state, double lr, double beta, int flags,
  *    pool-adjacent-violators on each chain, in fp32 (sample counts and sums are
  *    exact; fp64 would cost ~14x in the sequential chains), warm-started from the
  *    previous estimate's dual variables, stopped when a sweep moves no cell by
- *    more than tol x the largest cell mean.
+ *    more than tol x the largest cell mean.  The solution is constant on blocks of
+ *    cells, each at the count-weighted mean of its samples: one more sweep records
+ *    which cells the projections pool, and every block's value is then its mean
+ *    in fp64 from the exact cell sums (blocks that still break the order are
+ *    merged, in at most 32 rounds; if that does not settle, the fp32 values stand
+ *    and DBW_PSW_UNPOLISHED is raised).  The pooled column means and their PAVA
+ *    are fp64 too.
  *
  * The state is one opaque device buffer of dbw_psw_bytes(n) bytes that starts
  * with this header (the offsets locate its arrays, for inspection):
@@ -423,7 +444,7 @@ int dbw_choose_b(dbw_state* state, double lr, double beta, int flags,
 typedef struct {
     int32_t n;          /* workers */
     int32_t h;          /* k_{t-1} (n before the first iteration) */
-    int32_t sweeps;     /* Dykstra sweeps of the last dbw_psw_estimate */
+    int32_t sweeps;     /* Dykstra sweeps of the last dbw_psw_estimate (the recording sweep not counted) */
     int32_t flags;      /* DBW_PSW_* bits, sticky */
     double vclock;      /* tau_t, the push-and-wait virtual clock */
     double unit;        /* value of one unit of the int64 cell sums (2^-32) */
@@ -439,8 +460,9 @@ typedef struct {
 
 #define DBW_PSW_NOT_CONVERGED 1 /* the last estimate stopped at max_sweeps */
 #define DBW_PSW_RANGE 2         /* a sample outside [0, 2^31) was clamped in the cell sums */
+#define DBW_PSW_UNPOLISHED 4    /* the exact block means did not settle: T^ is the fp32 fit */
 
-/* Bytes of the push-and-wait state for n workers (grows as n^2: 5.3 MB at n = 256, 84 MB at n = 1024). */
+/* Bytes of the push-and-wait state for n workers (grows as n^2: 6.0 MB at n = 256, 76 MB at n = 1024). */
 size_t dbw_psw_bytes(int n);
 
 /* All workers idle, no sample, tau = 0, h = n.  psw: 256-byte aligned device buffer. */

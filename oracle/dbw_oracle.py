@@ -249,11 +249,16 @@ def sgd_update(w, gbar, lr):
 
 
 # ============================================ Sect. 3.1: gradient statistics
-def row_sqnorms(G, mask):
-    """||g_j||^2 for the received rows j (NaN for rows not received)."""
+def row_sqnorms(G, mask, all_rows=False):
+    """||g_j||^2 for the received rows j (NaN for rows not received).
+
+    R12: the statistics of Eq. (10) use the k received rows only.  With
+    ``all_rows`` the norm of every row is reported as well (the rows the PS did
+    not receive included); none of them enters a statistic."""
     G = np.asarray(G, dtype=np.float64)
     r = np.full(G.shape[0], np.nan)
-    for j in np.flatnonzero(np.asarray(mask)):
+    rows = range(G.shape[0]) if all_rows else np.flatnonzero(np.asarray(mask))
+    for j in rows:
         r[j] = float(np.dot(G[j], G[j]))
     return r
 

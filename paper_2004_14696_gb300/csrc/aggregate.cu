@@ -13,6 +13,11 @@
 // are processed UNROLL at a time, and the next batch's 128-bit loads are issued
 // before the current batch is reduced.
 //
+// With DBW_ALL_ROW_NORMS the rows the mask leaves out are read too, after the
+// received ones, for their squared norms only (Sect. 3.1's statistics still use
+// the received rows alone); that adds (n - k) d * 4 bytes.  It is a separate
+// instantiation of the kernel, so the default one is unchanged.
+//
 // Numerics.  Per column the warp keeps s1 = sum (x - c) and s2 = sum (x - c)^2 in
 // fp32 with the shift c = the column's value in the first received row, so that
 // sum_j (x_j - mean)^2 = s2 - s1^2 / k does not cancel.  Per-row squared norms
@@ -52,13 +57,16 @@ __device__ __forceinline__ double warp_sum_d(double v) {
     return v;
 }
 
+// kAllRows: also the squared norms of the rows the mask leaves out (DBW_ALL_ROW_NORMS).
+template <bool kAllRows>
 __global__ void __launch_bounds__(kThreads, 3) aggregate_kernel(
     const float* __restrict__ G, int64_t ld, int n, int64_t d, const uint8_t* __restrict__ mask,
     float lr, float* __restrict__ w, float* __restrict__ gbar, double* __restrict__ partials,
     int nblocks) {
     extern __shared__ double smem_d[];
     double* rowacc = smem_d;                           // [kWarps][n] fp64 row-norm pieces
-    int* sel = reinterpret_cast<int*>(smem_d + (size_t)kWarps * n);   // [n] received rows
+    // [n] rows in reading order: the received ones, then (kAllRows) the others
+    int* sel = reinterpret_cast<int*>(smem_d + (size_t)kWarps * n);
     __shared__ int k_s;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -67,10 +75,16 @@ __global__ void __launch_bounds__(kThreads, 3) aggregate_kernel(
         for (int j = 0; j < n; ++j)
             if (mask[j]) sel[k++] = j;
         k_s = k;
+        if (kAllRows) {
+            int r = k;
+            for (int j = 0; j < n; ++j)
+                if (!mask[j]) sel[r++] = j;
+        }
     }
     for (int i = tid; i < kWarps * n; i += kThreads) rowacc[i] = 0.0;
     __syncthreads();
     const int k = k_s;
+    const int64_t hdr_flags = kAllRows ? DBW_ALL_ROW_NORMS : 0;
     if (k == 0) {   // nothing received: leave w untouched, record empty pieces
         double* vals = partials + kPartialsHeader + (n + 2);
         for (int q = tid; q < n + 2; q += kThreads) vals[(int64_t)q * nblocks + blockIdx.x] = 0.0;
@@ -79,10 +93,13 @@ __global__ void __launch_bounds__(kThreads, 3) aggregate_kernel(
             hdr[0] = kPartialsMagic;
             hdr[1] = nblocks;
             hdr[2] = n;
-            hdr[3] = 0;
+            hdr[3] = hdr_flags;
         }
         return;
     }
+    // rows read per chunk: the k received ones (their statistics), then with kAllRows
+    // the n - k others (their squared norms only)
+    const int nrows = kAllRows ? n : k;
     const float inv_k = 1.0f / (float)k;
     double* myrow = rowacc + (size_t)warp * n;
 
@@ -130,29 +147,31 @@ __global__ void __launch_bounds__(kThreads, 3) aggregate_kernel(
 #pragma unroll
         for (int u = 0; u < UNROLL; ++u) {
             const int p = 1 + u;
-            const float* rowp = G + (int64_t)sel[p < k ? p : 0] * ld;
+            const float* rowp = G + (int64_t)sel[p < nrows ? p : 0] * ld;
 #pragma unroll
             for (int v = 0; v < VEC; ++v) {
                 const int64_t col = col0 + v * 128;
-                xn[u][v] = (p < k && inb[v]) ? ldg_stream(reinterpret_cast<const float4*>(rowp + col)) : c[v];
+                xn[u][v] = (p < nrows && inb[v]) ? ldg_stream(reinterpret_cast<const float4*>(rowp + col))
+                                                 : c[v];
             }
         }
-        for (int p0 = 1; p0 < k; p0 += UNROLL) {
+        for (int p0 = 1; p0 < nrows; p0 += UNROLL) {
             float4 x[UNROLL][VEC];
 #pragma unroll
             for (int u = 0; u < UNROLL; ++u)
 #pragma unroll
                 for (int v = 0; v < VEC; ++v) x[u][v] = xn[u][v];
-            if (p0 + UNROLL < k) {
+            if (p0 + UNROLL < nrows) {
 #pragma unroll
                 for (int u = 0; u < UNROLL; ++u) {
                     const int p = p0 + UNROLL + u;
-                    const float* rowp = G + (int64_t)sel[p < k ? p : 0] * ld;
+                    const float* rowp = G + (int64_t)sel[p < nrows ? p : 0] * ld;
 #pragma unroll
                     for (int v = 0; v < VEC; ++v) {
                         const int64_t col = col0 + v * 128;
-                        xn[u][v] = (p < k && inb[v]) ? ldg_stream(reinterpret_cast<const float4*>(rowp + col))
-                                                     : c[v];
+                        xn[u][v] = (p < nrows && inb[v])
+                                       ? ldg_stream(reinterpret_cast<const float4*>(rowp + col))
+                                       : c[v];
                     }
                 }
             }
@@ -169,16 +188,18 @@ __global__ void __launch_bounds__(kThreads, 3) aggregate_kernel(
                         if (col + 2 >= d) xv.z = c[v].z;
                         if (col + 3 >= d) xv.w = c[v].w;
                     }
-                    const float dx0 = xv.x - c[v].x, dx1 = xv.y - c[v].y;
-                    const float dx2 = xv.z - c[v].z, dx3 = xv.w - c[v].w;
-                    s1[v].x += dx0; s1[v].y += dx1; s1[v].z += dx2; s1[v].w += dx3;
-                    s2[v].x = fmaf(dx0, dx0, s2[v].x); s2[v].y = fmaf(dx1, dx1, s2[v].y);
-                    s2[v].z = fmaf(dx2, dx2, s2[v].z); s2[v].w = fmaf(dx3, dx3, s2[v].w);
+                    if (!kAllRows || p < k) {   // rows read past the received ones add no statistics
+                        const float dx0 = xv.x - c[v].x, dx1 = xv.y - c[v].y;
+                        const float dx2 = xv.z - c[v].z, dx3 = xv.w - c[v].w;
+                        s1[v].x += dx0; s1[v].y += dx1; s1[v].z += dx2; s1[v].w += dx3;
+                        s2[v].x = fmaf(dx0, dx0, s2[v].x); s2[v].y = fmaf(dx1, dx1, s2[v].y);
+                        s2[v].z = fmaf(dx2, dx2, s2[v].z); s2[v].w = fmaf(dx3, dx3, s2[v].w);
+                    }
                     rn = fmaf(xv.x, xv.x, rn); rn = fmaf(xv.y, xv.y, rn);
                     rn = fmaf(xv.z, xv.z, rn); rn = fmaf(xv.w, xv.w, rn);
                 }
                 rn = warp_sum(rn);
-                if (p < k && lane == 0) myrow[p] += (double)rn;
+                if (p < nrows && lane == 0) myrow[p] += (double)rn;
             }
         }
         // column epilogue: mean, SGD step, deviation sum, ||g_t||^2
@@ -232,8 +253,8 @@ __global__ void __launch_bounds__(kThreads, 3) aggregate_kernel(
     double* vals = partials + kPartialsHeader + (n + 2);
     for (int q = tid; q < n; q += kThreads) vals[(int64_t)q * nblocks + blockIdx.x] = 0.0;
     __syncthreads();
-    // rows are indexed by received position in rowacc; scatter them to worker ids
-    for (int p = tid; p < k; p += kThreads) {
+    // rows are indexed by reading position in rowacc; scatter them to worker ids
+    for (int p = tid; p < nrows; p += kThreads) {
         double s = 0.0;
         for (int wv = 0; wv < kWarps; ++wv) s += rowacc[(size_t)wv * n + p];
         vals[(int64_t)sel[p] * nblocks + blockIdx.x] = s;
@@ -251,7 +272,7 @@ __global__ void __launch_bounds__(kThreads, 3) aggregate_kernel(
             hdr[0] = kPartialsMagic;
             hdr[1] = nblocks;
             hdr[2] = n;
-            hdr[3] = 0;
+            hdr[3] = hdr_flags;
         }
     }
 }
@@ -263,7 +284,8 @@ size_t agg_smem_bytes(int n) { return (size_t)kWarps * n * sizeof(double) + (siz
 AggGeometry agg_geometry(int n, int64_t d) {
     AggGeometry g;
     int per_sm = 0;
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, aggregate_kernel, kThreads, agg_smem_bytes(n));
+    // both instantiations have the same launch shape; the default one sets the grid
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, aggregate_kernel<false>, kThreads, agg_smem_bytes(n));
     if (per_sm < 1) per_sm = 1;
     const int64_t nchunks = (d + kChunkCols - 1) / kChunkCols;
     int64_t blocks = (int64_t)sm_count() * per_sm;
@@ -276,17 +298,28 @@ AggGeometry agg_geometry(int n, int64_t d) {
     return g;
 }
 
-cudaError_t launch_aggregate(const float* G, int64_t ld, int n, int64_t d, const uint8_t* mask,
-                             float lr, float* w, float* gbar, double* partials, const AggGeometry& g,
-                             cudaStream_t st) {
+namespace {
+template <bool kAllRows>
+cudaError_t launch_aggregate_t(const float* G, int64_t ld, int n, int64_t d, const uint8_t* mask, float lr,
+                               float* w, float* gbar, double* partials, const AggGeometry& g, cudaStream_t st) {
     const size_t smem = agg_smem_bytes(n);
     if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(aggregate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)smem);
+        cudaError_t e = cudaFuncSetAttribute(aggregate_kernel<kAllRows>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
     }
-    aggregate_kernel<<<g.blocks, kThreads, smem, st>>>(G, ld, n, d, mask, lr, w, gbar, partials, g.blocks);
+    aggregate_kernel<kAllRows><<<g.blocks, kThreads, smem, st>>>(G, ld, n, d, mask, lr, w, gbar, partials,
+                                                                 g.blocks);
     return cudaGetLastError();
+}
+}  // namespace
+
+cudaError_t launch_aggregate(const float* G, int64_t ld, int n, int64_t d, const uint8_t* mask,
+                             float lr, float* w, float* gbar, int flags, double* partials, const AggGeometry& g,
+                             cudaStream_t st) {
+    if (flags & DBW_ALL_ROW_NORMS)
+        return launch_aggregate_t<true>(G, ld, n, d, mask, lr, w, gbar, partials, g, st);
+    return launch_aggregate_t<false>(G, ld, n, d, mask, lr, w, gbar, partials, g, st);
 }
 
 }  // namespace dbw

@@ -29,6 +29,8 @@ int fail(int code, const char* fmt, ...) {
     return code;
 }
 
+void clear_error() { g_err[0] = 0; }
+
 int check_launch(const char* what) {
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(DBW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
@@ -85,7 +87,7 @@ extern "C" {
 
 const char* dbw_last_error_string(void) { return g_err; }
 
-int dbw_abi_version(void) { return 1; }
+int dbw_abi_version(void) { return 2; }
 
 int64_t dbw_param_count(int num_layers, const int32_t* widths) {
     if (!widths || num_layers < 1 || num_layers > DBW_LMAX) return -1;
@@ -149,10 +151,11 @@ size_t dbw_aggregate_partials_bytes(int n, int64_t d) {
 }
 
 int dbw_aggregate_update(const float* G, int64_t ld, int n, int64_t d, const uint8_t* mask, float lr, float* w,
-                         float* gbar, double* partials, size_t partials_bytes, void* stream) {
+                         float* gbar, int flags, double* partials, size_t partials_bytes, void* stream) {
     g_err[0] = 0;
     Call call("dbw_aggregate_update", as_stream(stream));
     if (!G || !mask || !w || !partials) return fail(DBW_EINVAL, "dbw_aggregate_update: NULL pointer argument");
+    if (flags & ~DBW_ALL_ROW_NORMS) return fail(DBW_EINVAL, "dbw_aggregate_update: unknown flags");
     if (n < 1 || n > DBW_NMAX) return fail(DBW_EINVAL, "dbw_aggregate_update: n must be in [1, %d]", DBW_NMAX);
     if (d < 1) return fail(DBW_EINVAL, "dbw_aggregate_update: d must be >= 1");
     if (ld < d || ld % 4 != 0) return fail(DBW_EALIGN, "dbw_aggregate_update: ld must be >= d and a multiple of 4");
@@ -163,7 +166,7 @@ int dbw_aggregate_update(const float* G, int64_t ld, int n, int64_t d, const uin
     const AggGeometry g = agg_geometry(n, d);
     if (partials_bytes < g.bytes)
         return fail(DBW_EINVAL, "dbw_aggregate_update: partials %zu bytes < %zu needed", partials_bytes, g.bytes);
-    cudaError_t e = launch_aggregate(G, ld, n, d, mask, lr, w, gbar, partials, g, as_stream(stream));
+    cudaError_t e = launch_aggregate(G, ld, n, d, mask, lr, w, gbar, flags, partials, g, as_stream(stream));
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_aggregate_update: %s", cudaGetErrorString(e));
     return call.done(DBW_OK);
 }

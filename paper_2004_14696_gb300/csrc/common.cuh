@@ -11,6 +11,8 @@ namespace dbw {
 
 // Records a message for dbw_last_error_string() and returns ``code``.
 int fail(int code, const char* fmt, ...);
+// Empties dbw_last_error_string() of the calling thread (every entry point starts with it).
+void clear_error();
 // Maps a pending launch error to DBW_ECUDA (with its text), else DBW_OK.
 int check_launch(const char* what);
 // Number of SMs of the current device (cached per device).
@@ -53,8 +55,9 @@ struct AggGeometry {
     size_t bytes;         // total partials bytes
 };
 AggGeometry agg_geometry(int n, int64_t d);
+// flags: 0 or DBW_ALL_ROW_NORMS
 cudaError_t launch_aggregate(const float* G, int64_t ld, int n, int64_t d, const uint8_t* mask,
-                             float lr, float* w, float* gbar, double* partials,
+                             float lr, float* w, float* gbar, int flags, double* partials,
                              const AggGeometry& g, cudaStream_t st);
 
 // Estimator (estimator.cu)
@@ -90,7 +93,7 @@ int launch_received_grads(int L, const int32_t* widths, int prec, float* w, int6
                           float* gbar, float* loss, double* partials, void* ws, size_t ws_bytes, cudaStream_t st);
 
 // Partials buffer layout shared by aggregate.cu, grads_tc.cu and estimator.cu:
-//   int64 header[4] = {magic, blocks, n, reserved}
+//   int64 header[4] = {magic, blocks, n, flags (DBW_ALL_ROW_NORMS when every row's norm is in)}
 //   double sums[n + 2]              reduced totals (written by dbw_grad_stats)
 //   double vals[(n + 2) * blocks]   per-block pieces, by quantity: vals[q * blocks + blk]
 //                                   q < n: ||g_q||^2, q = n: SS, q = n + 1: ||g_t||^2

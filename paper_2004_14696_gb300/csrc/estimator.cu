@@ -131,8 +131,11 @@ __global__ void __launch_bounds__(1024) grad_stats_kernel(
     }
     // Sect. 3.2: every arrival is observed, S[r] accumulates the r-th order statistic
     for (int r = tid; r < n; r += blockDim.x) st->S[r] = st->S[r] + tsorted[r];
-    if (row_sqnorm)
-        for (int j = tid; j < n; j += blockDim.x) row_sqnorm[j] = mask[j] ? sums[j] : CUDART_NAN;
+    if (row_sqnorm) {
+        // the partials header says whether the rows the mask left out were read too
+        const bool all_rows = (reinterpret_cast<const int64_t*>(sums - kPartialsHeader)[3] & DBW_ALL_ROW_NORMS) != 0;
+        for (int j = tid; j < n; j += blockDim.x) row_sqnorm[j] = (mask[j] || all_rows) ? sums[j] : CUDART_NAN;
+    }
 }
 
 // T_ext (nullable): time estimates T^_k = T_ext[k-1] instead of S[k-1] / c; NaN in

@@ -21,8 +21,10 @@ DBW_OK, DBW_EINVAL, DBW_EALIGN, DBW_ECUDA, DBW_EUNSUPPORTED = 0, -1, -2, -3, -4
 PREC_FP32, PREC_BF16 = 0, 1
 NMAX, DMAX, LMAX = 1024, 64, 8
 CHOOSE_BLIND = 1
+ALL_ROW_NORMS = 1
+NOALLOC_SCRATCH_BYTES = 4 << 20   # DBW_NOALLOC_SCRATCH_BYTES
 FLAG_K1, FLAG_L_SKIPPED, FLAG_EMPTY_MASK, FLAG_BAD_STATE = 1, 2, 4, 8
-PSW_NOT_CONVERGED, PSW_RANGE = 1, 2
+PSW_NOT_CONVERGED, PSW_RANGE, PSW_UNPOLISHED = 1, 2, 4
 STAT_K, STAT_SS, STAT_GBAR_SQ, STAT_V, STAT_N, STAT_F, STAT_L, STAT_FLAGS, STAT_VCLOCK = range(9)
 STATS_LEN = 9
 PARTIALS_MAGIC = 0x44425750415254
@@ -73,8 +75,8 @@ _SIGS = {
                                 _vp, _sz, _vp]),
     "dbw_select_fastest": (_i32, [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp]),
     "dbw_aggregate_partials_bytes": (_sz, [_i32, _i64]),
-    "dbw_aggregate_update": (_i32, [_vp, _i64, _i32, _i64, _vp, _f32, _vp, _vp, _vp, _sz, _vp]),
-    "dbw_aggregate_update_noalloc": (_i32, [_vp, _i64, _i32, _i64, _vp, _f32, _vp, _vp, _vp, _vp]),
+    "dbw_aggregate_update": (_i32, [_vp, _i64, _i32, _i64, _vp, _f32, _vp, _vp, _i32, _vp, _sz, _vp]),
+    "dbw_aggregate_update_noalloc": (_i32, [_vp, _i64, _i32, _i64, _vp, _f32, _vp, _vp, _i32, _vp, _vp]),
     "dbw_received_grads_workspace_bytes": (_sz, [_i32, _vp, _i32, _i32, _i32]),
     "dbw_received_partials_bytes": (_sz, [_i32]),
     "dbw_received_grads_update": (_i32, [_i32, _vp, _i32, _vp, _i64, _vp, _i64, _vp, _vp, _i32, _i32, _vp, _f32,
@@ -275,20 +277,20 @@ def dbw_select_fastest(times, b, order, mask, tsorted, k_out=None, stream=None):
     _check("dbw_select_fastest", rc)
 
 
-def dbw_aggregate_update(G, n, d, mask, lr, w, partials, gbar=None, stream=None):
+def dbw_aggregate_update(G, n, d, mask, lr, w, partials, gbar=None, stream=None, flags=0):
     rc = lib().dbw_aggregate_update(
         _ptr(G, torch.float32, "G"), G.shape[1], n, d, _ptr(mask, torch.uint8, "mask"), float(lr),
-        _ptr(w, torch.float32, "w"), _ptr(gbar, torch.float32, "gbar", nullable=True),
+        _ptr(w, torch.float32, "w"), _ptr(gbar, torch.float32, "gbar", nullable=True), int(flags),
         _ptr(partials, torch.uint8, "partials"), partials.numel(), _stream(stream))
     _check("dbw_aggregate_update", rc)
 
 
-def dbw_aggregate_update_noalloc(G, n, d, mask, lr, w, sums_out, gbar=None, stream=None):
+def dbw_aggregate_update_noalloc(G, n, d, mask, lr, w, sums_out, gbar=None, stream=None, flags=0):
     """dbw_aggregate_update without caller scratch (for callers that cannot allocate);
     writes the reduced totals to sums_out [n + 2] fp64."""
     rc = lib().dbw_aggregate_update_noalloc(
         _ptr(G, torch.float32, "G"), G.shape[1], n, d, _ptr(mask, torch.uint8, "mask"), float(lr),
-        _ptr(w, torch.float32, "w"), _ptr(gbar, torch.float32, "gbar", nullable=True),
+        _ptr(w, torch.float32, "w"), _ptr(gbar, torch.float32, "gbar", nullable=True), int(flags),
         _ptr(sums_out, torch.float64, "sums_out"), _stream(stream))
     _check("dbw_aggregate_update_noalloc", rc)
 

@@ -84,9 +84,26 @@ def test_host_validation_rejects_before_launch(lib):
     assert b"NULL" in lib.dbw_last_error_string()
     assert lib.dbw_select_fastest(16, 0, 16, 16, 16, 16, null, null) == dbw.DBW_EINVAL
     assert lib.dbw_select_fastest(16, dbw.NMAX + 1, 16, 16, 16, 16, null, null) == dbw.DBW_EINVAL
-    assert lib.dbw_aggregate_update(256, 6, 4, 5, 256, C.c_float(0.1), 256, null, 256, 1 << 20, null) == dbw.DBW_EALIGN
-    assert lib.dbw_aggregate_update(260, 8, 4, 5, 256, C.c_float(0.1), 256, null, 256, 1 << 20, null) == dbw.DBW_EALIGN
-    assert lib.dbw_aggregate_update(256, 8, 0, 5, 256, C.c_float(0.1), 256, null, 256, 1 << 20, null) == dbw.DBW_EINVAL
+    assert lib.dbw_aggregate_update(256, 6, 4, 5, 256, C.c_float(0.1), 256, null, 0, 256, 1 << 20,
+                                    null) == dbw.DBW_EALIGN
+    assert lib.dbw_aggregate_update(260, 8, 4, 5, 256, C.c_float(0.1), 256, null, 0, 256, 1 << 20,
+                                    null) == dbw.DBW_EALIGN
+    assert lib.dbw_aggregate_update(256, 8, 0, 5, 256, C.c_float(0.1), 256, null, 0, 256, 1 << 20,
+                                    null) == dbw.DBW_EINVAL
+    # an unknown flag bit is refused, for both aggregation entry points
+    assert lib.dbw_aggregate_update(256, 8, 4, 5, 256, C.c_float(0.1), 256, null, 2, 256, 1 << 20,
+                                    null) == dbw.DBW_EINVAL
+    assert b"flags" in lib.dbw_last_error_string()
+    assert lib.dbw_aggregate_update_noalloc(256, 8, 4, 5, 256, C.c_float(0.1), 256, null, 6, 256,
+                                            null) == dbw.DBW_EINVAL
+    # every entry point starts from an empty error text
+    assert lib.dbw_param_count(1, null) == -1
+    assert lib.dbw_aggregate_update_noalloc(256, 8, dbw.NMAX + 1, 5, 256, C.c_float(0.1), 256, null, 0, 256,
+                                            null) == dbw.DBW_EINVAL
+    assert lib.dbw_last_error_string() != b""
+    assert lib.dbw_aggregate_update_noalloc(256, 6, 4, 5, 256, C.c_float(0.1), 256, null, 0, 256,
+                                            null) == dbw.DBW_EALIGN
+    assert b"ld" in lib.dbw_last_error_string() and b"n must" not in lib.dbw_last_error_string()
     assert lib.dbw_state_init(256, 4, 0, null) == dbw.DBW_EINVAL
     assert lib.dbw_state_init(256, 4, dbw.DMAX + 1, null) == dbw.DBW_EINVAL
     assert lib.dbw_choose_b(256, C.c_double(0.1), C.c_double(0.5), 0, 256, null, null) == dbw.DBW_EINVAL

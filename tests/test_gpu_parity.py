@@ -109,14 +109,14 @@ AGG_CASES = [(1, 5, 0), (2, 7, 1), (5, 3, 2), (16, 1000, 0), (16, 1000, 4), (16,
              (64, 12345, 16), (256, 4099, 0), (256, 4099, 255), (7, 256 * 37 + 1, 3), (3, 100003, 1)]
 
 
-def run_agg(G, w, times, b, lr, loss=None, gbar=True):
+def run_agg(G, w, times, b, lr, loss=None, gbar=True, flags=0):
     n, ld = G.shape
     d = w.shape[0]
     sel = gpu_select(times, b)
     Gd, wd, maskd = dev(G), dev(w), dev(sel["mask"])
     part = torch.empty(dbw.dbw_aggregate_partials_bytes(n, d), dtype=torch.uint8, device="cuda")
     gb = torch.empty(d, dtype=torch.float32, device="cuda") if gbar else None
-    dbw.dbw_aggregate_update(Gd, n, d, maskd, lr, wd, part, gb)
+    dbw.dbw_aggregate_update(Gd, n, d, maskd, lr, wd, part, gb, flags=flags)
     state = dbw.new_state(n, 5)
     stats = torch.empty(dbw.STATS_LEN, dtype=torch.float64, device="cuda")
     rn = torch.empty(n, dtype=torch.float64, device="cuda")
@@ -147,6 +147,27 @@ def test_aggregate_parity(n, d, b):
     r = O.row_sqnorms(Gd, mask)
     assert np.array_equal(np.isnan(rn), np.isnan(r))
     assert_close_rows(rn[~np.isnan(r)], r[~np.isnan(r)], RTOL_FP32, "row norms")
+
+
+@pytest.mark.parametrize("n,d,b", [(2, 7, 1), (16, 1000, 4), (16, 1000, 15), (64, 12345, 16), (256, 4099, 0),
+                                   (256, 4099, 255), (7, 256 * 37 + 1, 3), (3, 100003, 2)])
+def test_aggregate_all_row_norms(n, d, b):
+    """DBW_ALL_ROW_NORMS (R12): the rows the mask leaves out are read for their
+    squared norms, against the oracle; g_t, w_{t+1}, SS, ||g_t||^2 and the received
+    rows' norms are bit for bit those of the default call (the received rows go
+    through the same arithmetic in the same order)."""
+    G, w, times = agg_case(n, d, seed=2000 + n + d, b=b, mean=0.3)
+    lr = 0.05
+    _, w0, g0, s0, rn0 = run_agg(G, w, times, b, lr)
+    _, w1, g1, s1, rn1 = run_agg(G, w, times, b, lr, flags=dbw.ALL_ROW_NORMS)
+    assert np.array_equal(w0, w1) and np.array_equal(g0, g1)
+    assert same_f64(s0, s1)
+    _, mask, _ = O.select_fastest(times, b)
+    m = mask.astype(bool)
+    assert np.array_equal(rn0[m], rn1[m]) and np.all(np.isnan(rn0[~m]))
+    r = O.row_sqnorms(G[:, :d], mask, all_rows=True)
+    assert np.all(np.isfinite(rn1))
+    assert_close_rows(rn1, r, RTOL_FP32, "every row's squared norm")
 
 
 def test_aggregate_is_permutation_invariant_on_gpu():

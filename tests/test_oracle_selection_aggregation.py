@@ -122,6 +122,19 @@ def test_deviation_identity_with_row_norms():
     assert np.all(np.isnan(r[mask == 0]))
 
 
+def test_row_norms_of_every_row_closed_form():
+    """R12 with every row's norm: row j filled with +-(j+1) has ||g_j||^2 = d (j+1)^2,
+    received or not; the received rows' values are those of the default form."""
+    n, d = 6, 40
+    signs = np.where(np.random.default_rng(11).random((n, d)) < 0.5, -1.0, 1.0)
+    G = signs * (np.arange(n) + 1.0)[:, None]
+    mask = np.array([1, 0, 0, 1, 1, 0], dtype=np.uint8)
+    full = O.row_sqnorms(G, mask, all_rows=True)
+    assert np.array_equal(full, d * (np.arange(n) + 1.0) ** 2)
+    part = O.row_sqnorms(G, mask)
+    assert np.array_equal(part[mask == 1], full[mask == 1]) and np.all(np.isnan(part[mask == 0]))
+
+
 @pytest.mark.parametrize("k", [2, 3, 8])
 def test_variance_estimator_unbiased_and_second_moment(k):
     """Eq. (10) is unbiased (E V^+ = d sigma^2) and Eq. (8): E||g_t||^2 = ||mu||^2 + V/k."""
