@@ -11,10 +11,13 @@
 // dbw_aggregate_update writes into caller memory are written here into one
 // file-scope device array of fixed size (kScratchBytes).  Every GPU that loads
 // libdbw holds this array until the process exits.  All calls on a device share
-// it and it keeps whatever the last call wrote; nothing in it has to start at
-// zero, because each call overwrites every value it later reads.  Two calls
-// whose work overlaps on the GPU (different streams without ordering between
-// them) race on the array and corrupt each other's sums.
+// it and it keeps whatever the last call wrote.  Each call first clears the
+// array's header (cudaMemsetAsync on the call's stream, which allocates
+// nothing) and the aggregation kernel overwrites every other value the
+// reduction later reads; so if the aggregation does not run, the reduction
+// finds no valid header and writes NaN instead of the previous call's totals.
+// Two calls whose work overlaps on the GPU (different streams without ordering
+// between them) race on the array and corrupt each other's sums.
 //
 // Set-up: host code cannot use the array's name as a device address, so the
 // first call on each device asks the runtime for the array's device address
@@ -23,6 +26,8 @@
 // capture begins.
 //
 // This entry point calls no cudaMalloc, cudaFree or other allocating routine.
+#include <math_constants.h>
+
 #include <mutex>
 
 #include "common.cuh"
@@ -59,11 +64,16 @@ int scratch_address(void** out) {
 }
 
 // sums_out[q] = total of quantity q over the per-block pieces, in the same fixed
-// order dbw_grad_stats uses (256 strided partial sums, then a pairwise tree).
+// order dbw_grad_stats uses (256 strided partial sums, then a pairwise tree).  A
+// header that the aggregation of this call did not write gives NaN.
 constexpr int kRed = 256;
 __global__ void __launch_bounds__(kRed) reduce_to_sums_kernel(const double* __restrict__ partials, int n,
                                                               double* __restrict__ sums_out) {
     const int64_t* hdr = reinterpret_cast<const int64_t*>(partials);
+    if (hdr[0] != kPartialsMagic || hdr[2] != n || hdr[1] < 1 || hdr[1] > (1 << 20)) {
+        if (threadIdx.x == 0) sums_out[blockIdx.x] = CUDART_NAN;
+        return;
+    }
     const int blocks = (int)hdr[1];
     const double* vals = partials + kPartialsHeader + (n + 2) + (int64_t)blockIdx.x * blocks;
     __shared__ double red[kRed];
@@ -85,10 +95,13 @@ __global__ void __launch_bounds__(kRed) reduce_to_sums_kernel(const double* __re
 using namespace dbw;
 
 extern "C" int dbw_aggregate_update_noalloc(const float* G, int64_t ld, int n, int64_t d, const uint8_t* mask,
-                                            float lr, float* w, float* gbar, double* sums_out, void* stream) {
+                                            float lr, float* w, float* gbar, int flags, double* sums_out,
+                                            void* stream) {
+    clear_error();
     Call call("dbw_aggregate_update_noalloc", as_stream(stream));
     if (!G || !mask || !w || !sums_out)
         return fail(DBW_EINVAL, "dbw_aggregate_update_noalloc: NULL pointer argument");
+    if (flags & ~DBW_ALL_ROW_NORMS) return fail(DBW_EINVAL, "dbw_aggregate_update_noalloc: unknown flags");
     if (n < 1 || n > DBW_NMAX)
         return fail(DBW_EINVAL, "dbw_aggregate_update_noalloc: n must be in [1, %d]", DBW_NMAX);
     if (d < 1) return fail(DBW_EINVAL, "dbw_aggregate_update_noalloc: d must be >= 1");
@@ -109,7 +122,9 @@ extern "C" int dbw_aggregate_update_noalloc(const float* G, int64_t ld, int n, i
     if (rc) return rc;
     double* partials = static_cast<double*>(scratch);
     cudaStream_t st = as_stream(stream);
-    cudaError_t e = launch_aggregate(G, ld, n, d, mask, lr, w, gbar, partials, g, st);
+    cudaError_t e = cudaMemsetAsync(partials, 0, kPartialsHeader * sizeof(int64_t), st);
+    if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_aggregate_update_noalloc: %s", cudaGetErrorString(e));
+    e = launch_aggregate(G, ld, n, d, mask, lr, w, gbar, flags, partials, g, st);
     if (e != cudaSuccess) return fail(DBW_ECUDA, "dbw_aggregate_update_noalloc: %s", cudaGetErrorString(e));
     reduce_to_sums_kernel<<<n + 2, kRed, 0, st>>>(partials, n, sums_out);
     e = cudaGetLastError();
