@@ -26,6 +26,8 @@ STREAM_INDEX = 4
 STREAM_TIMES = 5
 STREAM_GRADS = 6
 STREAM_PICK = 7
+STREAM_GRAD_COLS = 8
+GRAD_COL_CHUNK = 1 << 16
 
 BASE_SEED = 2004146960
 
@@ -164,6 +166,34 @@ def gradient_matrix(seed: int, n: int, d: int, ld: int, mean: float = 0.0,
         G[i, :d] = mean + std * g.standard_normal(d, dtype=np.float32)
     G[:, d:] = np.nan
     return G
+
+
+def gradient_columns(seed: int, rows, c0: int, c1: int, threads: int = 1) -> np.ndarray:
+    """Columns ``[c0, c1)`` of the given rows of a synthetic gradient matrix, entries
+    N(0,1) drawn in fp32 and returned as fp64 ``[len(rows), c1 - c0]``.  Column chunk q
+    (``GRAD_COL_CHUNK`` columns) of row i comes from its own generator
+    ``(seed, STREAM_GRAD_COLS, i, q)``, so any column range of any row can be drawn on
+    its own, in any order, with the same values.  ``threads`` > 1 draws rows in
+    parallel (numpy releases the GIL while it fills an array)."""
+    rows = [int(i) for i in rows]
+    q0, q1 = c0 // GRAD_COL_CHUNK, (c1 + GRAD_COL_CHUNK - 1) // GRAD_COL_CHUNK
+    out = np.empty((len(rows), c1 - c0), dtype=np.float64)
+
+    def fill(r):
+        i = rows[r]
+        for q in range(q0, q1):
+            a, b = max(c0, q * GRAD_COL_CHUNK), min(c1, (q + 1) * GRAD_COL_CHUNK)
+            block = rng(seed, STREAM_GRAD_COLS, i, q).standard_normal(GRAD_COL_CHUNK, dtype=np.float32)
+            out[r, a - c0:b - c0] = block[a - q * GRAD_COL_CHUNK:b - q * GRAD_COL_CHUNK]
+
+    if threads > 1:
+        from concurrent.futures import ThreadPoolExecutor
+        with ThreadPoolExecutor(threads) as ex:
+            list(ex.map(fill, range(len(rows))))
+    else:
+        for r in range(len(rows)):
+            fill(r)
+    return out
 
 
 def round_up(x: int, m: int) -> int:
