@@ -1,14 +1,32 @@
 """Helpers shared by the GPU parity tests (no method arithmetic here)."""
 import math
+import os
 
 import numpy as np
 
 RTOL_FP32 = 1e-5    # fp32 GEMM / fp32 accumulation paths
 RTOL_BF16 = 2e-2    # bf16 GEMM operands with fp32 accumulation
 # bf16 elementwise outliers: at most this fraction of a worker's entries may exceed
-# 2e-2 of their error scale, and none by more than this factor
-BF16_OUTLIER_FRACTION = 1e-5
+# 2e-2 of their error scale (at least one entry), and none by more than this factor.
+# Set at twice the most measured on GB300 (24 of 54.4M entries, 4.4e-7, in one
+# worker of the 4096-wide model; worst 2.06x).
+BF16_OUTLIER_FRACTION = 9e-7
 BF16_OUTLIER_FACTOR = 4.0
+# ReLU decisions the GPU takes differently from the oracle (each one certified
+# ambiguous, R13): at most this fraction of a worker's decisions in any hidden layer,
+# or RELU_FLIP_FLOOR of them.  Twice the most measured on GB300: 45 of 131,072
+# decisions (3.4e-4) in the 4096-wide model, 2 in a layer of a small model.
+RELU_FLIP_FRACTION = 7e-4
+RELU_FLIP_FLOOR = 4
+
+# What the acceptance rules above actually took, one record per compared worker or
+# vector, printed at the end of the session (tests/conftest.py): ReLU decisions taken
+# from the GPU per hidden layer, and entries beyond 2e-2 of their error scale.
+ACCEPTANCE = []
+
+
+def _current_test():
+    return os.environ.get("PYTEST_CURRENT_TEST", "?").split(" ")[0]
 
 
 def param_blocks(widths):
@@ -104,6 +122,15 @@ def oracle_rows_with_decisions(widths, w, X, y, B, bf16, workers, gpu_active=Non
                                                 f"differ from the oracle's outside rounding of 0 "
                                                 f"(largest |Z|/scale {rel.max():.3g})")
                 flips.append(diff)
+            counts = [int(f.sum()) for f in flips]
+            sizes = [int(f.size) for f in flips]
+            ACCEPTANCE.append({"test": _current_test(), "kind": "relu", "worker": int(i), "bf16": bool(bf16),
+                               "flips": counts, "decisions": sizes})
+            if RELU_FLIP_FRACTION is not None:
+                for h, (c, sz) in enumerate(zip(counts, sizes)):
+                    assert c <= max(RELU_FLIP_FLOOR, RELU_FLIP_FRACTION * sz), (
+                        f"worker {i} layer {h}: {c} of {sz} ReLU decisions taken from the GPU, above the cap "
+                        f"{RELU_FLIP_FRACTION:g} of them")
             if any(f.any() for f in flips):
                 g, _, gm = O.worker_grads(widths, w, Xi, yi, 1, B, bf16, relu_flip=flips, return_magnitude=True)
         out[i] = (g[0], float(l[0]), gm[0])
@@ -124,8 +151,11 @@ def assert_bf16_close(x, ref, scale, blocks, rtol, what):
         assert num <= rtol * den, f"{what} tensor [{a},{b}): normwise relative error {num / den:.3g}"
     ratio = np.abs(x - r) / (rtol * scale)
     nbad = int((ratio > 1.0).sum())
+    ACCEPTANCE.append({"test": _current_test(), "kind": "outliers", "what": what, "outliers": nbad,
+                       "entries": int(x.size), "worst": float(ratio.max())})
     assert nbad <= max(1, int(BF16_OUTLIER_FRACTION * x.size)) and ratio.max() <= BF16_OUTLIER_FACTOR, (
         f"{what}: {nbad} of {x.size} entries beyond 2e-2 of their scale, worst {ratio.max():.3g}x")
+    return nbad
 
 
 def assert_worker_grads_match(G_gpu, loss_gpu, widths, w, X, y, B, bf16, workers, rtol, gpu_active=None,
@@ -192,3 +222,65 @@ def _bad_entries(x, r, rtol, blocks):
         seg = r2[a:b]
         scale[a:b] = np.sqrt(np.mean(seg * seg))
     return ~(np.abs(np.asarray(x, dtype=np.float64) - r2) <= rtol * (np.abs(r2) + scale))
+
+
+# ----------------------------------------------------------- oracle rows in worker processes
+# The full-size received-form check needs the oracle's Eq. (2) row of every received
+# worker (54.4M entries each on the largest workload).  The rows are formed in a pool of
+# spawned processes (one BLAS thread each); every process keeps only what the check
+# compares: sampled entries, norms, losses and the running sum of its workers' rows.
+_POOL_STATE = {}
+
+
+def _pool_init(widths, seed, bf16, entries, tensor_of_entry, blocks):
+    from paper_2004_14696_gb300 import inputs
+    _POOL_STATE.update(widths=tuple(widths), bf16=bf16, entries=np.asarray(entries),
+                       tensor_of_entry=np.asarray(tensor_of_entry), blocks=blocks,
+                       w=inputs.kaiming_uniform_params(seed, widths).astype(np.float64))
+
+
+def _pool_rows(task):
+    """Oracle rows of a chunk of workers (their minibatches X, y and the GPU's ReLU
+    decisions on their rows); returns per worker (loss, ||g_j||^2, g_j at the sampled
+    entries, the bf16 error scale there), the chunk's sum of rows and the acceptance
+    records."""
+    X, y, B, acts = task
+    st = _POOL_STATE
+    widths, blocks, ent = st["widths"], st["blocks"], st["entries"]
+    n = X.shape[0] // B
+    total = None
+    per = []
+    base = len(ACCEPTANCE)
+    for i in range(n):
+        rows = oracle_rows_with_decisions(widths, st["w"], X[i * B:(i + 1) * B], y[i * B:(i + 1) * B], B,
+                                          st["bf16"], [0], [a[i * B:(i + 1) * B] for a in acts])
+        g, loss, gm = rows[0]
+        rms = np.array([np.sqrt(np.mean(g[a:b] ** 2)) for (a, b) in blocks])
+        scale = np.maximum(gm[ent], np.abs(g[ent]) + rms[st["tensor_of_entry"]])
+        per.append((loss, float(g @ g), g[ent].copy(), scale))
+        total = g.copy() if total is None else total + g
+        del rows, g, gm
+    return per, total, ACCEPTANCE[base:]
+
+
+def oracle_rows_in_pool(widths, seed, bf16, entries, tensor_of_entry, blocks, tasks, procs=None):
+    """Run _pool_rows over ``tasks`` in spawned processes; returns the list of results."""
+    import multiprocessing as mp
+    from concurrent.futures import ProcessPoolExecutor
+    procs = procs or min(len(tasks), os.cpu_count() or 1)
+    keep = {k: os.environ.get(k) for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS")}
+    for k in keep:
+        os.environ[k] = "1"          # the spawned children start with one BLAS thread each
+    try:
+        with ProcessPoolExecutor(procs, mp_context=mp.get_context("spawn"), initializer=_pool_init,
+                                 initargs=(widths, seed, bf16, entries, tensor_of_entry, blocks)) as ex:
+            out = list(ex.map(_pool_rows, tasks))
+    finally:
+        for k, v in keep.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+    for (_, _, recs) in out:
+        ACCEPTANCE.extend(recs)
+    return out
