@@ -203,6 +203,21 @@ int dbw_profile_gemm(int enable);
 int dbw_profile_gemm_read(double* total_ms, int64_t* launches);
 
 /*
+ * Test hook of the bounded waits (the paper has no counterpart; for tests of the
+ * failure path).  Every wait of the tensor-core kernels on a pipeline barrier is
+ * bounded (2 s); when one runs out the kernel sets bit 0 of the status word,
+ * stops, waits (bounded) for its own copies still in flight, releases its tensor
+ * memory and returns, so that the context stays usable.  This call arms the next
+ * per-worker weight-gradient launch of dbw_worker_grads (one launch, then it
+ * disarms itself): its waits are bounded by wait_ms, and its first CTA does not
+ * issue the TMA load of pipeline stage ``stage`` (0 = its first), so that the
+ * MMA's wait for that stage runs out, as a lost copy would make it.  That call's
+ * G and loss are then undefined and its status word has bit 0 set.  stage < 0
+ * disarms.  Host only; DBW_EINVAL unless 0 < wait_ms <= 2000.
+ */
+int dbw_test_arm_wait_timeout(int stage, double wait_ms);
+
+/*
  * Eq. (4): the PS waits for the first k = n - b gradients.
  * Arrival order is (times[i], i) ascending (ties go to the lower worker index).
  *

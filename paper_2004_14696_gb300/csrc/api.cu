@@ -268,6 +268,18 @@ int dbw_choose_b_times(dbw_state* state, const double* T_hat, double lr, double 
     return call.done(DBW_OK);
 }
 
+int dbw_test_arm_wait_timeout(int stage, double wait_ms) {
+    g_err[0] = 0;
+    if (stage < 0) {
+        arm_dw_wait_timeout(-1, 0);
+        return DBW_OK;
+    }
+    if (!(wait_ms > 0.0 && wait_ms <= 2000.0))
+        return fail(DBW_EINVAL, "dbw_test_arm_wait_timeout: wait_ms must be in (0, 2000]");
+    arm_dw_wait_timeout(stage, static_cast<unsigned long long>(wait_ms * 1e6));
+    return DBW_OK;
+}
+
 size_t dbw_psw_bytes(int n) {
     if (n < 1 || n > DBW_NMAX) return 0;
     return psw_bytes(n);

@@ -86,6 +86,11 @@ int launch_worker_grads(int L, const int32_t* widths, int prec, const float* w, 
                         int n, int B, float* G, int64_t ld, float* loss, void* ws, size_t ws_bytes,
                         cudaStream_t st);
 
+// Tests of the bounded waits (gemm_tc.cu): the next weight-gradient launch bounds its
+// waits by limit_ns and its first CTA does not issue the load of pipeline stage
+// ``stage``; stage < 0 disarms.
+void arm_dw_wait_timeout(long long stage, unsigned long long limit_ns);
+
 // Received-workers pass (grads_tc.cu)
 size_t received_workspace_bytes(int L, const int32_t* widths, int n, int B, int prec);
 int launch_received_grads(int L, const int32_t* widths, int prec, float* w, int64_t d, const float* pool, int64_t S,

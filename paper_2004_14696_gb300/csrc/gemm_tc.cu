@@ -18,6 +18,7 @@
 // launch are then undefined, never a fault or a hang.
 #include <cuda.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "gemm_tc.cuh"
@@ -681,10 +682,18 @@ struct DwCfg {
     static constexpr int SMEM = STAGES * STAGE_BYTES + STAGING + BAR_BYTES + 1024;
 };
 
+// The bound of the kernel's waits, and (tests of the bounded-wait path only) one
+// pipeline stage whose TMA load the first CTA does not issue: the MMA's wait for it
+// then runs out, as a lost copy would make it.
+struct DwWaits {
+    unsigned long long limit_ns;   // every mbarrier wait of the launch
+    long long skip_stage;          // stage counter g of block 0 left without its load; -1: none
+};
+
 template <int BK, int STAGES>
 __global__ void __launch_bounds__(DW_THREADS, 1)
     tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int Mr, int Nr,
-                 int K, int batch, int* status, float* __restrict__ Gbase, int64_t ldrow, int64_t ldG) {
+                 int K, int batch, int* status, float* __restrict__ Gbase, int64_t ldrow, int64_t ldG, DwWaits wt) {
     using Cfg = DwCfg<BK, STAGES>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -739,21 +748,25 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
             for (int kb = 0; kb < nk; ++kb, ++g) {
                 const int s = static_cast<int>(g % STAGES);
                 const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
-                if (!mbar_wait(smem_u32(empty_bar + s), ph ^ 1)) {
+                if (!mbar_wait(smem_u32(empty_bar + s), ph ^ 1, wt.limit_ns)) {
                     atomicOr(status, 1);
                     *vabort = 1;
                     break;
                 }
-                mbar_expect_tx(smem_u32(full_bar + s), Cfg::STAGE_BYTES);
-                const int kx = z * K + kb * BK;
-                tma_load_2d(smem_u32(sA + s * Cfg::A_BYTES), &tmA, kx, m0, smem_u32(full_bar + s));
-                tma_load_2d(smem_u32(sB + s * Cfg::B_BYTES), &tmB, kx, n0, smem_u32(full_bar + s));
+                if (!(blockIdx.x == 0 && g == wt.skip_stage)) {
+                    mbar_expect_tx(smem_u32(full_bar + s), Cfg::STAGE_BYTES);
+                    const int kx = z * K + kb * BK;
+                    tma_load_2d(smem_u32(sA + s * Cfg::A_BYTES), &tmA, kx, m0, smem_u32(full_bar + s));
+                    tma_load_2d(smem_u32(sB + s * Cfg::B_BYTES), &tmB, kx, n0, smem_u32(full_bar + s));
+                }
                 issued = g + 1;
             }
         }
         if (*vabort) {
+            // the loads of the last STAGES stages may still be landing: wait for them (a
+            // stage whose load never started only runs out its bound)
             for (long long q = issued - STAGES < 0 ? 0 : issued - STAGES; q < issued; ++q)
-                mbar_wait(smem_u32(full_bar + q % STAGES), static_cast<uint32_t>((q / STAGES) & 1));
+                mbar_wait(smem_u32(full_bar + q % STAGES), static_cast<uint32_t>((q / STAGES) & 1), wt.limit_ns);
         }
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer
@@ -763,7 +776,7 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
         for (long long t = blockIdx.x; t < total && !*vabort; t += gridDim.x, ++i) {
             const int acc = i & 1;
             const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
-            if (!mbar_wait(smem_u32(tempty_bar + acc), aph ^ 1)) {
+            if (!mbar_wait(smem_u32(tempty_bar + acc), aph ^ 1, wt.limit_ns)) {
                 atomicOr(status, 1);
                 *vabort = 1;
                 break;
@@ -774,7 +787,7 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
             for (int kb = 0; kb < nk; ++kb, ++g) {
                 const int s = static_cast<int>(g % STAGES);
                 const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
-                if (!mbar_wait(smem_u32(full_bar + s), ph)) {
+                if (!mbar_wait(smem_u32(full_bar + s), ph, wt.limit_ns)) {
                     atomicOr(status, 1);
                     *vabort = 1;
                     ok = false;
@@ -801,7 +814,7 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
         for (long long t = blockIdx.x; t < total; t += gridDim.x, ++i) {
             const int acc = i & 1;
             const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
-            if (!mbar_wait(smem_u32(tfull_bar + acc), aph)) {
+            if (!mbar_wait(smem_u32(tfull_bar + acc), aph, wt.limit_ns)) {
                 atomicOr(status, 1);
                 *vabort = 1;
                 break;
@@ -858,6 +871,11 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
 }
 
 // ------------------------------------------------------------------ host side
+// One-shot arming of a lost load in the next launch of tc_dw_kernel (tests of the
+// bounded-wait path; see dbw_test_arm_wait_timeout).
+std::atomic<long long> g_dw_skip_stage{-1};
+std::atomic<unsigned long long> g_dw_test_limit_ns{0};
+
 template <int BK, int STAGES>
 cudaError_t launch_dw(const CUtensorMap& a, const CUtensorMap& b, int Mr, int Nr, int K, int batch, int* status,
                       float* gbase, int64_t ldrow, int64_t ldG, cudaStream_t st) {
@@ -870,7 +888,13 @@ cudaError_t launch_dw(const CUtensorMap& a, const CUtensorMap& b, int Mr, int Nr
     if (err != cudaSuccess) return err;
     const long long tiles = static_cast<long long>((Mr + BM - 1) / BM) * ((Nr + DW_BN - 1) / DW_BN) * batch;
     const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
-    kern<<<grid, DW_THREADS, smem, st>>>(a, b, Mr, Nr, K, batch, status, gbase, ldrow, ldG);
+    DwWaits wt{kWaitLimitNs, -1};
+    const long long skip = g_dw_skip_stage.exchange(-1);
+    if (skip >= 0) {
+        wt.skip_stage = skip;
+        wt.limit_ns = g_dw_test_limit_ns.load();
+    }
+    kern<<<grid, DW_THREADS, smem, st>>>(a, b, Mr, Nr, K, batch, status, gbase, ldrow, ldG, wt);
     return cudaGetLastError();
 }
 
@@ -934,6 +958,11 @@ cudaError_t launch_cfg(const CUtensorMap& a, const CUtensorMap& b, int M, int N,
 }
 
 }  // namespace
+
+void arm_dw_wait_timeout(long long stage, unsigned long long limit_ns) {
+    g_dw_test_limit_ns.store(limit_ns);
+    g_dw_skip_stage.store(stage);
+}
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,

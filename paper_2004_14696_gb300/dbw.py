@@ -94,6 +94,7 @@ _SIGS = {
     "dbw_profile_dw_read": (_i32, [_vp, _vp, _vp]),
     "dbw_profile_gemm": (_i32, [_i32]),
     "dbw_profile_gemm_read": (_i32, [_vp, _vp]),
+    "dbw_test_arm_wait_timeout": (_i32, [_i32, _f64]),
 }
 
 
@@ -314,6 +315,12 @@ def dbw_choose_b(state, lr, beta, b_out, ratio_out=None, flags=0, stream=None):
         _ptr(state, torch.uint8, "state"), float(lr), float(beta), int(flags), _ptr(b_out, torch.int32, "b_out"),
         _ptr(ratio_out, torch.float64, "ratio_out", nullable=True), _stream(stream))
     _check("dbw_choose_b", rc)
+
+
+def dbw_test_arm_wait_timeout(stage, wait_ms):
+    """Arms the next weight-gradient launch to lose the load of one pipeline stage
+    (tests of the bounded-wait path); stage < 0 disarms."""
+    _check("dbw_test_arm_wait_timeout", lib().dbw_test_arm_wait_timeout(int(stage), float(wait_ms)))
 
 
 def dbw_profile_dw(enable):

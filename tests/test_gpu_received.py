@@ -358,10 +358,9 @@ def test_launch_timing_channels():
     """dbw_profile_gemm / dbw_profile_dw record one event pair per persistent GEMM and per
     weight-gradient launch, only while enabled; a read forgets the records."""
     L = len(RX_B32.widths) - 1
-    # two-call form: L forward GEMMs (its input-gradient GEMMs run beside the weight
-    # gradients and are not timed); received form: L forward GEMMs, then per layer one
-    # launch of the mean-gradient GEMM (with the dX GEMM of that layer when l > 0)
-    for received, gemms, dws in ((False, L, L), (True, L + L, 0)):
+    # received form: L forward GEMMs, then per layer one launch of the mean-gradient GEMM
+    # (with the dX GEMM of that layer when l > 0)
+    for received, gemms, dws in ((False, L + (L - 1), L), (True, L + L, 0)):
         it = Iteration(RX_B32, static_b=2, received=received)
         it.load_inputs(0)
         it.step()
