@@ -747,8 +747,9 @@ def extras():
     cfg[workloads.MLP3072.key] = {"two_call": iterate_case(workloads.MLP3072.key, 200, 10, graph=True),
                                   "received": iterate_case(workloads.MLP3072.key, 200, 10, received=True, graph=True)}
     from paper_2004_14696_gb300 import dbw
-    pts = [(256, 10 ** 8, 0, 0), (256, 10 ** 8, 64, 0), (256, 10 ** 8, 64, dbw.ALL_ROW_NORMS),
-           (64, 10 ** 7, 0, 0), (64, 10 ** 7, 16, 0)]
+    # the small matrix first: measured right after the 102 GB one it read slower
+    pts = [(64, 10 ** 7, 0, 0), (64, 10 ** 7, 16, 0),
+           (256, 10 ** 8, 0, 0), (256, 10 ** 8, 64, 0), (256, 10 ** 8, 64, dbw.ALL_ROW_NORMS)]
     cfg["aggregation_sweep"] = sweep_points(pts, reps=10)
     cfg["psw_fit"] = {str(n): psw_case(n, 60) for n in (16, 256)}
     return cfg
