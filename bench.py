@@ -53,18 +53,21 @@ from paper_2004_14696_gb300 import inputs, workloads  # noqa: E402
 METRIC = "simulated PS iterations/sec at n workers"
 UNIT = "iter/s"
 
-# dram bytes (read + write) of one aggregation launch from an ncu capture (n = 64,
-# d = 4e6, k = 48), as a ratio to the algorithmic bytes so that it scales to the
+# dram bytes (read + write) of one full-size aggregation launch from an ncu capture
+# (n = 256, d = 54,440,936, k = 142: 31.1411 GB read + 0.1717 GB written against
+# 31.3580 GB algorithmic), as a ratio to the algorithmic bytes so that it scales to the
 # bench's launches (traffic grows with k d); reported as null once aggregate.cu
 # differs from the source the counters were taken on.
-AGG_TRAFFIC = {"ratio_to_algorithmic": None, "source_sha256": None, "case": "n=64 d=4e6 k=48"}
+AGG_TRAFFIC = {"ratio_to_algorithmic": (31.141070 + 0.171713) / 31.357979,
+               "source_sha256": "1d5f6bb0b751a7ad2fae28b88999146db77319f34bc6ba9bcc4d5be0abfcec09",
+               "case": "n=256 d=54440936 k=142"}
 # dram bytes (read + write) of the per-worker weight-gradient launches of one
-# full-size step (ncu on mlp4096x3-1000_n256_B32): 4.2130 + 17.2599 + 17.2596 +
-# 17.2583 GB against 4.2778 + 3 x 17.3141 GB algorithmic; keyed to the dW kernel's
+# full-size pass (ncu on mlp4096x3-1000_n256_B32): 4.2158 + 17.2505 + 17.2508 +
+# 17.2520 GB against 4.2778 + 3 x 17.3141 GB algorithmic; keyed to the dW kernel's
 # own source (dw_source_sha).
-DW_TRAFFIC = {"ratio_to_algorithmic": (4.2130 + 17.2599 + 17.2596 + 17.2583) / (4.2778 + 3 * 17.3141),
-              "source_sha256": "49652b56fb1338974566dcb78b1b940bb43688a603dfa846f820898c31d62839",
-              "case": "mlp4096x3-1000_n256_B32, one step"}
+DW_TRAFFIC = {"ratio_to_algorithmic": (4.2158 + 17.2505 + 17.2508 + 17.2520) / (4.2778 + 3 * 17.3141),
+              "source_sha256": "bafb8a813d2b51c8c7e1921e5fa40487cfd5f74fde82f3e96748fb7521c6d77b",
+              "case": "mlp4096x3-1000_n256_B32, one pass"}
 
 CASES = ("aggregate", "sweep", "grads", "received", "psw", "iterate")
 
@@ -552,7 +555,7 @@ def aggregate_case(n, d, b, reps, flags=0, seed=workloads.AGG_SEED, G=None):
     seeded generator: input generation only) with the n - b fastest of Exp(1) times."""
     import torch
     from paper_2004_14696_gb300 import dbw
-    ld = inputs.round_up(d, 4)
+    ld = inputs.round_up(d, 32)          # rows start on 128-byte boundaries, as in the workloads
     g = torch.Generator(device="cuda")
     g.manual_seed(seed + n)
     if G is None:
@@ -583,7 +586,7 @@ def sweep_points(points, reps):
     import torch
     out = []
     for (n, d), group in _group_points(points).items():
-        ld = inputs.round_up(d, 4)
+        ld = inputs.round_up(d, 32)
         g = torch.Generator(device="cuda")
         g.manual_seed(workloads.AGG_SEED + n)
         G = torch.randn((n, ld), generator=g, device="cuda", dtype=torch.float32)

@@ -682,18 +682,20 @@ struct DwCfg {
     static constexpr int SMEM = STAGES * STAGE_BYTES + STAGING + BAR_BYTES + 1024;
 };
 
-// The bound of the kernel's waits, and (tests of the bounded-wait path only) one
-// pipeline stage whose TMA load the first CTA does not issue: the MMA's wait for it
-// then runs out, as a lost copy would make it.
+// Tests of the bounded-wait path (the kTest instantiation, launched only when armed):
+// the bound of the kernel's waits, and one pipeline stage whose TMA load the first CTA
+// does not issue, so that the MMA's wait for it runs out as a lost copy would make it.
+// The production instantiation ignores these: its waits are bounded by kWaitLimitNs.
 struct DwWaits {
     unsigned long long limit_ns;   // every mbarrier wait of the launch
     long long skip_stage;          // stage counter g of block 0 left without its load; -1: none
 };
 
-template <int BK, int STAGES>
+template <int BK, int STAGES, bool kTest = false>
 __global__ void __launch_bounds__(DW_THREADS, 1)
     tc_dw_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int Mr, int Nr,
                  int K, int batch, int* status, float* __restrict__ Gbase, int64_t ldrow, int64_t ldG, DwWaits wt) {
+    const uint64_t wait_ns = kTest ? wt.limit_ns : kWaitLimitNs;
     using Cfg = DwCfg<BK, STAGES>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -748,12 +750,12 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
             for (int kb = 0; kb < nk; ++kb, ++g) {
                 const int s = static_cast<int>(g % STAGES);
                 const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
-                if (!mbar_wait(smem_u32(empty_bar + s), ph ^ 1, wt.limit_ns)) {
+                if (!mbar_wait(smem_u32(empty_bar + s), ph ^ 1, wait_ns)) {
                     atomicOr(status, 1);
                     *vabort = 1;
                     break;
                 }
-                if (!(blockIdx.x == 0 && g == wt.skip_stage)) {
+                if (!(kTest && blockIdx.x == 0 && g == wt.skip_stage)) {
                     mbar_expect_tx(smem_u32(full_bar + s), Cfg::STAGE_BYTES);
                     const int kx = z * K + kb * BK;
                     tma_load_2d(smem_u32(sA + s * Cfg::A_BYTES), &tmA, kx, m0, smem_u32(full_bar + s));
@@ -766,7 +768,7 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
             // the loads of the last STAGES stages may still be landing: wait for them (a
             // stage whose load never started only runs out its bound)
             for (long long q = issued - STAGES < 0 ? 0 : issued - STAGES; q < issued; ++q)
-                mbar_wait(smem_u32(full_bar + q % STAGES), static_cast<uint32_t>((q / STAGES) & 1), wt.limit_ns);
+                mbar_wait(smem_u32(full_bar + q % STAGES), static_cast<uint32_t>((q / STAGES) & 1), wait_ns);
         }
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer
@@ -776,7 +778,7 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
         for (long long t = blockIdx.x; t < total && !*vabort; t += gridDim.x, ++i) {
             const int acc = i & 1;
             const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
-            if (!mbar_wait(smem_u32(tempty_bar + acc), aph ^ 1, wt.limit_ns)) {
+            if (!mbar_wait(smem_u32(tempty_bar + acc), aph ^ 1, wait_ns)) {
                 atomicOr(status, 1);
                 *vabort = 1;
                 break;
@@ -787,7 +789,7 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
             for (int kb = 0; kb < nk; ++kb, ++g) {
                 const int s = static_cast<int>(g % STAGES);
                 const uint32_t ph = static_cast<uint32_t>((g / STAGES) & 1);
-                if (!mbar_wait(smem_u32(full_bar + s), ph, wt.limit_ns)) {
+                if (!mbar_wait(smem_u32(full_bar + s), ph, wait_ns)) {
                     atomicOr(status, 1);
                     *vabort = 1;
                     ok = false;
@@ -814,7 +816,7 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
         for (long long t = blockIdx.x; t < total; t += gridDim.x, ++i) {
             const int acc = i & 1;
             const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
-            if (!mbar_wait(smem_u32(tfull_bar + acc), aph, wt.limit_ns)) {
+            if (!mbar_wait(smem_u32(tfull_bar + acc), aph, wait_ns)) {
                 atomicOr(status, 1);
                 *vabort = 1;
                 break;
@@ -880,7 +882,14 @@ template <int BK, int STAGES>
 cudaError_t launch_dw(const CUtensorMap& a, const CUtensorMap& b, int Mr, int Nr, int K, int batch, int* status,
                       float* gbase, int64_t ldrow, int64_t ldG, cudaStream_t st) {
     using Cfg = DwCfg<BK, STAGES>;
-    auto kern = tc_dw_kernel<BK, STAGES>;
+    DwWaits wt{kWaitLimitNs, -1};
+    const long long skip = g_dw_skip_stage.exchange(-1);
+    const bool test = skip >= 0;
+    if (test) {
+        wt.skip_stage = skip;
+        wt.limit_ns = g_dw_test_limit_ns.load();
+    }
+    auto kern = test ? tc_dw_kernel<BK, STAGES, true> : tc_dw_kernel<BK, STAGES, false>;
     // each CTA holds all 512 TMEM columns: ask for enough shared memory that a
     // second CTA can never be resident on the same SM (it would wait in tcgen05.alloc)
     const int smem = Cfg::SMEM > 120 * 1024 ? Cfg::SMEM : 120 * 1024;
@@ -888,12 +897,6 @@ cudaError_t launch_dw(const CUtensorMap& a, const CUtensorMap& b, int Mr, int Nr
     if (err != cudaSuccess) return err;
     const long long tiles = static_cast<long long>((Mr + BM - 1) / BM) * ((Nr + DW_BN - 1) / DW_BN) * batch;
     const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
-    DwWaits wt{kWaitLimitNs, -1};
-    const long long skip = g_dw_skip_stage.exchange(-1);
-    if (skip >= 0) {
-        wt.skip_stage = skip;
-        wt.limit_ns = g_dw_test_limit_ns.load();
-    }
     kern<<<grid, DW_THREADS, smem, st>>>(a, b, Mr, Nr, K, batch, status, gbase, ldrow, ldG, wt);
     return cudaGetLastError();
 }
