@@ -759,7 +759,10 @@ def extras():
 
 
 # ====================================================================== CPU oracle
-REF_AGG_SLICES = 128    # the oracle's aggregation runs on 1/128 of the columns per step
+def ref_agg_slices(wl):
+    """Column slices of the oracle's aggregation sample: the whole width when n d is small
+    (up to 2^24 entries), else about 2^24 entries per slice, at most 128 slices."""
+    return int(min(128, max(1, -(-wl.n * wl.d // (1 << 24)))))
 
 
 def oracle_step_seconds(wl, t, pool, labels, w, agg=True, threads=1):
@@ -769,8 +772,8 @@ def oracle_step_seconds(wl, t, pool, labels, w, agg=True, threads=1):
     Sample: the Eq. (2) gradients of 2 of the n workers (each worker's gradient is an
     independent Eq. (2) over its own B samples; scaled by n/2), selection and the
     estimator in full, and the aggregation + statistics of every worker's row over
-    column slice t mod 128 (d/128 columns: n distinct seeded rows drawn outside the
-    timed part; scaled by 128).  k = n: the estimator's choice from a fresh state
+    column slice t mod S of S = ref_agg_slices(wl) (n distinct seeded rows drawn outside
+    the timed part; scaled by S).  k = n: the estimator's choice from a fresh state
     (k_0 = n, Sect. 3), kept for every sampled step."""
     from oracle import dbw_oracle as O
     n, B = wl.n, wl.B
@@ -789,15 +792,16 @@ def oracle_step_seconds(wl, t, pool, labels, w, agg=True, threads=1):
     t_sel = time.perf_counter() - t0
     t_agg = 0.0
     if agg:
-        s = t % REF_AGG_SLICES
-        c0, c1 = s * wl.d // REF_AGG_SLICES, (s + 1) * wl.d // REF_AGG_SLICES
+        S = ref_agg_slices(wl)
+        s = t % S
+        c0, c1 = s * wl.d // S, (s + 1) * wl.d // S
         Gs = inputs.gradient_columns(wl.seed, range(n), c0, c1, threads=threads)
         t0 = time.perf_counter()
         gbar = O.aggregate(Gs, mask)
         O.sgd_update(w[c0:c1], gbar, wl.lr)
         O.deviation_sumsq(Gs, mask, gbar)
         O.row_sqnorms(Gs, mask)
-        t_agg = (time.perf_counter() - t0) * REF_AGG_SLICES
+        t_agg = (time.perf_counter() - t0) * S
         del Gs
     return t_grad + t_sel + t_agg, {"grads_s": t_grad, "select_estimator_s": t_sel, "aggregation_s": t_agg}
 
@@ -810,10 +814,10 @@ def _oracle_inputs(wl):
 
 
 def _oracle_sample_text(wl, steps):
+    S = ref_agg_slices(wl)
     return ("%d sampled iterations, each: Eq. (2) for 2 of the %d workers (x%d), selection and estimator in full, "
             "aggregation + statistics of all %d distinct seeded rows over one 1/%d column slice (x%d; the slices "
-            "of the steps differ), k = n; fp64 numpy" % (steps, wl.n, wl.n // 2, wl.n, REF_AGG_SLICES,
-                                                        REF_AGG_SLICES))
+            "of the steps differ), k = n; fp64 numpy" % (steps, wl.n, wl.n // 2, wl.n, S, S))
 
 
 def run_reference(args, rank, world):
@@ -834,7 +838,7 @@ def run_reference(args, rank, world):
     sec = float(np.mean(per))
     cores = int(os.environ.get("OPENBLAS_NUM_THREADS", os.cpu_count() or 1))
     value = 1.0 / sec
-    extrap = {"grads": wl.n / 2.0, "aggregation": float(REF_AGG_SLICES), "select_estimator": 1.0}
+    extrap = {"grads": wl.n / 2.0, "aggregation": float(ref_agg_slices(wl)), "select_estimator": 1.0}
     mean_parts = {k2: float(np.mean([p[k2] for p in parts])) for k2 in parts[0]}
     return {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True,
@@ -862,7 +866,7 @@ def cpu_baseline_for(wl, budget_s=25.0):
     cores = int(os.environ.get("OPENBLAS_NUM_THREADS", os.cpu_count() or 1))
     return {"value": 1.0 / float(np.mean(per)), "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": _oracle_sample_text(wl, len(per)),
-            "extrapolated": {"grads": wl.n / 2.0, "aggregation": float(REF_AGG_SLICES), "select_estimator": 1.0},
+            "extrapolated": {"grads": wl.n / 2.0, "aggregation": float(ref_agg_slices(wl)), "select_estimator": 1.0},
             "seconds_per_step_by_part": {k2: float(np.mean([p[k2] for p in parts])) for k2 in parts[0]}}
 
 
