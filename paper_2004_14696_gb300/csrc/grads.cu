@@ -63,7 +63,10 @@ __global__ void cast_bf16_kernel(const float* __restrict__ w, int64_t d, __nv_bf
 
 // ------------------------------------------------------------------ SIMT GEMM
 // C[m, n] = sum_k A(m, k) B(k, n) over a 128 x 128 tile per CTA, 16-deep K
-// slices staged in shared memory as fp32, 8 x 8 outputs per thread.
+// slices staged in shared memory as fp32, 8 x 8 outputs per thread.  Two shared
+// buffers: the next slice's global loads go to registers while the current slice
+// is multiplied, then to the other buffer (every output still adds its products
+// in increasing k).
 //   A_K: A(m,k) = A[m*lda + k]   else A(m,k) = A[k*lda + m]
 //   B_K: B(k,n) = B[n*ldb + k]   else B(k,n) = B[k*ldb + n]
 // blockIdx.z is a batch index (offsets batchA / batchB).
@@ -77,8 +80,8 @@ template <typename T, bool A_K, bool B_K, class Epi, bool SPLIT>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(int M, int N, int K, const T* __restrict__ A, int64_t lda,
                                                         int64_t batchA, const T* __restrict__ B, int64_t ldb,
                                                         int64_t batchB, Epi epi, int kps, float* __restrict__ part) {
-    __shared__ __align__(16) float As[BK][BM];
-    __shared__ __align__(16) float Bs[BK][BN];
+    __shared__ __align__(16) float As[2][BK][BM];
+    __shared__ __align__(16) float Bs[2][BK][BN];
     const int z = blockIdx.z;
     if (!SPLIT) {
         A += (int64_t)z * batchA;
@@ -94,32 +97,55 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(int M, int N, int K, con
 #pragma unroll
         for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
 
-    for (int k0 = kbeg; k0 < kend; k0 += BK) {
+    constexpr int LA = BM * BK / 256, LB = BN * BK / 256;   // elements per thread and slice
+    float ra[LA], rb[LB];
+    // global -> registers: the slice starting at k0 (element e of the tile is thread e % 256's)
+    auto load = [&](int k0) {
 #pragma unroll
-        for (int e = tid; e < BM * BK; e += 256) {
+        for (int q = 0; q < LA; ++q) {
+            const int e = tid + q * 256;
             int mm, kk;
             if (A_K) { mm = e / BK; kk = e % BK; } else { kk = e / BM; mm = e % BM; }
             const int gm = m0 + mm, gk = k0 + kk;
-            float v = 0.f;
-            if (gm < M && gk < kend) v = to_f<T>(A_K ? A[(int64_t)gm * lda + gk] : A[(int64_t)gk * lda + gm]);
-            As[kk][mm] = v;
+            ra[q] = (gm < M && gk < kend) ? to_f<T>(A_K ? A[(int64_t)gm * lda + gk] : A[(int64_t)gk * lda + gm]) : 0.f;
         }
 #pragma unroll
-        for (int e = tid; e < BN * BK; e += 256) {
+        for (int q = 0; q < LB; ++q) {
+            const int e = tid + q * 256;
             int nn, kk;
             if (B_K) { nn = e / BK; kk = e % BK; } else { kk = e / BN; nn = e % BN; }
             const int gn = n0 + nn, gk = k0 + kk;
-            float v = 0.f;
-            if (gn < N && gk < kend) v = to_f<T>(B_K ? B[(int64_t)gn * ldb + gk] : B[(int64_t)gk * ldb + gn]);
-            Bs[kk][nn] = v;
+            rb[q] = (gn < N && gk < kend) ? to_f<T>(B_K ? B[(int64_t)gn * ldb + gk] : B[(int64_t)gk * ldb + gn]) : 0.f;
         }
-        __syncthreads();
+    };
+    // registers -> shared buffer ``buf``
+    auto store = [&](int buf) {
+#pragma unroll
+        for (int q = 0; q < LA; ++q) {
+            const int e = tid + q * 256;
+            if (A_K) As[buf][e % BK][e / BK] = ra[q]; else As[buf][e / BM][e % BM] = ra[q];
+        }
+#pragma unroll
+        for (int q = 0; q < LB; ++q) {
+            const int e = tid + q * 256;
+            if (B_K) Bs[buf][e % BK][e / BK] = rb[q]; else Bs[buf][e / BN][e % BN] = rb[q];
+        }
+    };
+    if (kbeg < kend) {
+        load(kbeg);
+        store(0);
+    }
+    __syncthreads();
+    int buf = 0;
+    for (int k0 = kbeg; k0 < kend; k0 += BK) {
+        const bool more = k0 + BK < kend;
+        if (more) load(k0 + BK);   // in flight while this slice is multiplied
 #pragma unroll
         for (int kk = 0; kk < BK; ++kk) {
-            const float4 a0 = *reinterpret_cast<const float4*>(&As[kk][ty * 4]);
-            const float4 a1 = *reinterpret_cast<const float4*>(&As[kk][64 + ty * 4]);
-            const float4 b0 = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
-            const float4 b1 = *reinterpret_cast<const float4*>(&Bs[kk][64 + tx * 4]);
+            const float4 a0 = *reinterpret_cast<const float4*>(&As[buf][kk][ty * 4]);
+            const float4 a1 = *reinterpret_cast<const float4*>(&As[buf][kk][64 + ty * 4]);
+            const float4 b0 = *reinterpret_cast<const float4*>(&Bs[buf][kk][tx * 4]);
+            const float4 b1 = *reinterpret_cast<const float4*>(&Bs[buf][kk][64 + tx * 4]);
             const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
             const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
@@ -127,7 +153,10 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(int M, int N, int K, con
 #pragma unroll
                 for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
         }
+        // the other buffer was last read before the previous barrier
+        if (more) store(buf ^ 1);
         __syncthreads();
+        buf ^= 1;
     }
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
