@@ -56,6 +56,10 @@ int tc_gemm(int kind, const __nv_bfloat16* A, int64_t lda, int64_t rowsA, int64_
 // or rejects the arguments.
 bool tc_make_map(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_k, int box_rows);
 
+// The same for a row-major fp32 matrix: box 32 (128 bytes, 128-byte swizzle) x box_rows;
+// ld a multiple of 4 and base 16-byte aligned.
+bool tc_make_map_f32(CUtensorMap* tm, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_rows);
+
 // True when tc_gemm can run this problem (alignment rules above).
 bool tc_shape_ok(int64_t lda, int64_t ldb, int K, int64_t kz, const void* A, const void* B);
 

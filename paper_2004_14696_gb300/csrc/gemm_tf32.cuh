@@ -1,0 +1,226 @@
+// fp32 GEMM on the tcgen05 tensor cores in three tf32 passes (3xTF32), for the fp32
+// workloads' forward GEMMs.  Internal header (templates on the epilogue).
+//
+// Every fp32 operand x is split into hi = x rounded to nearest tf32 (10 mantissa bits)
+// and lo = x - hi (exact in fp32, |lo| <= 2^-11 |x|), itself stored rounded to nearest
+// tf32, so that the tensor core reads both parts exactly.  Then
+// x y ~ hi_x hi_y + hi_x lo_y + lo_x hi_y: the dropped lo_x lo_y and the rounding of lo
+// are each at most 2^-22 of |x y|, and unbiased.
+//
+// The accumulation is split too, because the tensor core's fp32 accumulation is not
+// assumed to round to nearest: the hi.hi products of 32-deep K block kb go to TMEM
+// accumulator kb mod NMAIN, the two correction products of every block to one more
+// accumulator (its terms are 2^-11 of the others, so its own rounding is negligible),
+// and the epilogue adds the NMAIN + 1 partial sums in fp32, rounding to nearest.  Each
+// accumulator then takes about K / (8 NMAIN) MMA additions instead of 3 K / 8.
+//
+// One CTA per 128 x BN output tile (the single-CTA layout of tc_gemm_kernel): a TMA
+// producer thread, an MMA thread, four epilogue warps (one per 32-row TMEM lane
+// quarter).  A stage holds 32-deep K slices of A_hi, A_lo (128 rows) and B_hi, B_lo
+// (BN rows), 128-byte swizzled; its 4 K = 8 steps issue 3 MMAs each.  Every wait is
+// bounded (2 s); if one runs out, bit 0 of ``status`` is set and the tile is skipped.
+#pragma once
+
+#include "gemm_tc.cuh"
+#include "tc_ptx.cuh"
+
+namespace dbw {
+namespace tf32 {
+
+constexpr int BM = 128;
+constexpr int kThreads = 192;
+constexpr int BK = 32;   // fp32 elements per 128-byte row
+
+template <int BN, int STAGES, int NMAIN>
+struct Cfg {
+    static constexpr int A_BYTES = BM * BK * 4;    // one of A_hi / A_lo
+    static constexpr int B_BYTES = BN * BK * 4;    // one of B_hi / B_lo
+    static constexpr int STAGE_BYTES = 2 * A_BYTES + 2 * B_BYTES;
+    static constexpr int SMEM = STAGES * STAGE_BYTES + 256 + 1024;
+    static constexpr int ACC_COLS = (NMAIN + 1) * BN;   // NMAIN hi.hi accumulators, then the corrections
+    static constexpr int TMEM_COLS = ACC_COLS <= 32 ? 32 : ACC_COLS <= 64 ? 64 : ACC_COLS <= 128 ? 128
+                                   : ACC_COLS <= 256 ? 256 : 512;
+    static_assert(BN % 32 == 0 && BN >= 32 && BN <= 256, "BN: a multiple of 32 up to 256");
+    static_assert(ACC_COLS <= 512, "the accumulators exceed TMEM");
+};
+
+struct Operands {
+    CUtensorMap a_hi, a_lo, b_hi, b_lo;   // A [M, K], B [N, K], fp32 row-major, K contiguous
+};
+
+// hi / lo parts of a row-major fp32 matrix [rows, cols] (row stride lds) into two
+// matrices with row stride ldo.
+__global__ void split_kernel(const float* __restrict__ src, int rows, int cols, int64_t lds,
+                             float* __restrict__ hi, float* __restrict__ lo, int64_t ldo);
+
+template <int BN, int STAGES, int NMAIN, class Epi>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_kernel(const __grid_constant__ Operands op, int M, int N, int K, Epi epi, int* status) {
+    using C = Cfg<BN, STAGES, NMAIN>;
+    using namespace tcx;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    // stage s: A_hi, A_lo, B_hi, B_lo
+    auto part = [&](int s, int which) {
+        const int off = which < 2 ? which * C::A_BYTES : 2 * C::A_BYTES + (which - 2) * C::B_BYTES;
+        return smem + s * C::STAGE_BYTES + off;
+    };
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
+    uint64_t* empty_bar = full_bar + STAGES;
+    uint64_t* accum_bar = empty_bar + STAGES;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum_bar + 1);
+    int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
+    const int nk = (K + BK - 1) / BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(smem_u32(full_bar + s), 1);
+            mbar_init(smem_u32(empty_bar + s), 1);
+        }
+        mbar_init(smem_u32(accum_bar), 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tc_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
+        tc_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer
+        int issued = 0;
+        for (int kb = 0; kb < nk; ++kb) {
+            const int s = kb % STAGES;
+            const uint32_t ph = (kb / STAGES) & 1;
+            if (!mbar_wait(smem_u32(empty_bar + s), ph ^ 1)) {
+                atomicOr(status, 1);
+                atomicExch(abort_flag, 1);
+                break;
+            }
+            if (*reinterpret_cast<volatile int*>(abort_flag)) break;
+            const uint32_t fb = smem_u32(full_bar + s);
+            mbar_expect_tx(fb, C::STAGE_BYTES);
+            tma_load_2d(smem_u32(part(s, 0)), &op.a_hi, kb * BK, m0, fb);
+            tma_load_2d(smem_u32(part(s, 1)), &op.a_lo, kb * BK, m0, fb);
+            tma_load_2d(smem_u32(part(s, 2)), &op.b_hi, kb * BK, n0, fb);
+            tma_load_2d(smem_u32(part(s, 3)), &op.b_lo, kb * BK, n0, fb);
+            issued = kb + 1;
+        }
+        if (*reinterpret_cast<volatile int*>(abort_flag)) {
+            // this thread's copies that may still be in flight (the last STAGES issued)
+            for (int kb = issued - STAGES < 0 ? 0 : issued - STAGES; kb < issued; ++kb)
+                mbar_wait(smem_u32(full_bar + kb % STAGES), (kb / STAGES) & 1);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer: per K = 8 step hi.hi (accumulator kb mod NMAIN),
+        // hi.lo and lo.hi (the correction accumulator)
+        constexpr uint32_t idesc = instr_desc_tf32(BM, BN);
+        const uint32_t corr = tmem + NMAIN * BN;
+        for (int kb = 0; kb < nk; ++kb) {
+            const int s = kb % STAGES;
+            const uint32_t ph = (kb / STAGES) & 1;
+            if (!mbar_wait(smem_u32(full_bar + s), ph)) {
+                atomicOr(status, 1);
+                atomicExch(abort_flag, 1);
+                break;
+            }
+            tc_fence_after();
+            const uint32_t ah = smem_u32(part(s, 0)), al = smem_u32(part(s, 1));
+            const uint32_t bh = smem_u32(part(s, 2)), bl = smem_u32(part(s, 3));
+#pragma unroll
+            for (int kk = 0; kk < BK / 8; ++kk) {
+                const uint32_t o = kk * 32;   // 8 fp32 = 32 bytes of K per step
+                tc_mma_tf32(tmem + (kb % NMAIN) * BN, smem_desc(ah + o, 128), smem_desc(bh + o, 128), idesc,
+                            (kb >= NMAIN || kk > 0) ? 1u : 0u);
+                tc_mma_tf32(corr, smem_desc(ah + o, 128), smem_desc(bl + o, 128), idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                tc_mma_tf32(corr, smem_desc(al + o, 128), smem_desc(bh + o, 128), idesc, 1u);
+            }
+            tc_commit(smem_u32(empty_bar + s));   // frees the stage once these MMAs have read it
+        }
+        tc_commit(smem_u32(accum_bar));           // accumulator complete (or, after an abort, quiescent)
+    } else if (warp >= 2) {
+        // ---------------- epilogue: TMEM lane quarter q = rows m0 + 32 q ..
+        if (!mbar_wait(smem_u32(accum_bar), 0)) {
+            atomicOr(status, 1);
+        } else if (!*reinterpret_cast<volatile int*>(abort_flag)) {
+            tc_fence_after();
+            const int q = warp & 3;
+            const int row = m0 + q * 32 + lane;
+            const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16);
+            const int used = nk < NMAIN ? nk : NMAIN;   // hi.hi accumulators written
+#pragma unroll 1
+            for (int c = 0; c < BN / 32; ++c) {
+                const int nb = n0 + c * 32;
+                if (nb >= N) break;
+                float v[32];
+                uint32_t r[32];
+#pragma unroll
+                for (int j = 0; j < 32; ++j) v[j] = 0.f;
+#pragma unroll 1
+                for (int a = 0; a < used; ++a) {
+                    tc_ld_32cols(tbase + a * BN + c * 32, r);
+                    tc_wait_ld();
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] += u2f(r[j]);
+                }
+                if (nk > 0) {
+                    tc_ld_32cols(tbase + NMAIN * BN + c * 32, r);
+                    tc_wait_ld();
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] += u2f(r[j]);
+                }
+                if (row < M) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (nb + j < N) epi(0, row, nb + j, v[j]);
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tc_dealloc(tmem, C::TMEM_COLS);
+    }
+}
+
+constexpr int kBN = 64;
+constexpr int kStages = 4;
+constexpr int kMain = 7;   // (7 + 1) x 64 = 512 TMEM columns
+
+// Splits both operands into ws buffers (a_hi, a_lo: [M, lda2]; b_hi, b_lo: [N, ldb2],
+// lda2 = ldb2 = K rounded up to 4) and runs C = A B^T into ``epi``.  A [M, K] (row
+// stride lda) and B [N, K] (row stride ldb) are fp32 row-major.
+template <class Epi>
+cudaError_t run(int M, int N, int K, const float* A, int64_t lda, const float* B, int64_t ldb, float* a_hi,
+                float* a_lo, float* b_hi, float* b_lo, Epi epi, int* status, cudaStream_t st) {
+    const int64_t ld2 = (K + 3) / 4 * 4;
+    {
+        dim3 g((K + 127) / 128, M < 65535 ? M : 65535);
+        split_kernel<<<g, 128, 0, st>>>(A, M, K, lda, a_hi, a_lo, ld2);
+        dim3 gb((K + 127) / 128, N < 65535 ? N : 65535);
+        split_kernel<<<gb, 128, 0, st>>>(B, N, K, ldb, b_hi, b_lo, ld2);
+    }
+    Operands op;
+    if (!tc_make_map_f32(&op.a_hi, a_hi, M, K, ld2, BM) || !tc_make_map_f32(&op.a_lo, a_lo, M, K, ld2, BM) ||
+        !tc_make_map_f32(&op.b_hi, b_hi, N, K, ld2, kBN) || !tc_make_map_f32(&op.b_lo, b_lo, N, K, ld2, kBN))
+        return cudaErrorInvalidValue;
+    using C = Cfg<kBN, kStages, kMain>;
+    auto kern = gemm_kernel<kBN, kStages, kMain, Epi>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
+    dim3 grid((N + kBN - 1) / kBN, (M + BM - 1) / BM);
+    kern<<<grid, kThreads, C::SMEM, st>>>(op, M, N, K, epi, status);
+    return cudaGetLastError();
+}
+
+}  // namespace tf32
+}  // namespace dbw

@@ -13,13 +13,48 @@
 //              dZ_{l-1} = (dZ_l W_l) * 1[A_{l-1} > 0]      (ReLU'(0) = 0)
 //
 // GEMMs here are the SIMT path (fp32 FFMA on fp32 or bf16 operands), used for the
-// fp32 workloads and for bf16 shapes the tcgen05 pass (grads_tc.cu) does not take.
+// fp32 workloads and for bf16 shapes the tcgen05 pass (grads_tc.cu) does not take;
+// the fp32 workloads' large forward GEMMs run on the tensor cores in three tf32
+// passes instead (gemm_tf32.cuh), which keeps fp32 accuracy.
 #include <math.h>
 
 #include "common.cuh"
+#include "gemm_tf32.cuh"
 #include "grads.cuh"
 
 namespace dbw {
+
+namespace tf32 {
+// x rounded to the nearest tf32 value (10 mantissa bits; ties to even), for finite x; a
+// value that would round up past the largest finite float is truncated instead.
+__device__ __forceinline__ float round_tf32(float x) {
+    const uint32_t u = __float_as_uint(x);
+    const uint32_t r = (u + 0x0FFFu + ((u >> 13) & 1u)) & 0xFFFFE000u;
+    return ((r & 0x7F800000u) == 0x7F800000u) ? __uint_as_float(u & 0xFFFFE000u) : __uint_as_float(r);
+}
+
+// hi = x rounded to nearest tf32, lo = x - hi (exact) rounded to nearest tf32.  A value
+// that is not finite goes whole to hi (a NaN as the canonical quiet NaN), lo = 0.
+__global__ void split_kernel(const float* __restrict__ src, int rows, int cols, int64_t lds, float* __restrict__ hi,
+                             float* __restrict__ lo, int64_t ldo) {
+    for (int r = blockIdx.y; r < rows; r += gridDim.y) {
+        const float* s = src + (int64_t)r * lds;
+        for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < cols; c += gridDim.x * blockDim.x) {
+            const float x = s[c];
+            float h, l;
+            if (isfinite(x)) {
+                h = round_tf32(x);
+                l = round_tf32(x - h);
+            } else {
+                h = isnan(x) ? __uint_as_float(0x7FC00000u) : x;
+                l = 0.f;
+            }
+            hi[(int64_t)r * ldo + c] = h;
+            lo[(int64_t)r * ldo + c] = l;
+        }
+    }
+}
+}  // namespace tf32
 
 namespace {
 
@@ -362,14 +397,29 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
         const int fin = P.widths[l], fout = P.widths[l + 1];
         const T* W = wop + P.offW[l];
         const float* bias = w + P.offb[l];
+        const bool tc = sizeof(T) == 4 && P.tf32[l];
+        float* part[4] = {nullptr, nullptr, nullptr, nullptr};
+        if (tc) {
+            part[0] = reinterpret_cast<float*>(ws + P.off_ahi);
+            part[1] = reinterpret_cast<float*>(ws + P.off_alo);
+            part[2] = reinterpret_cast<float*>(ws + P.off_whi);
+            part[3] = reinterpret_cast<float*>(ws + P.off_wlo);
+        }
+        int* status = reinterpret_cast<int*>(ws);
+        auto fwd = [&](auto epi) {
+            if constexpr (sizeof(T) == 4) {
+                if (tc)
+                    return tf32::run(M, fout, fin, Ain, fin, W, fin, part[0], part[1], part[2], part[3], epi, status,
+                                     st);
+            }
+            return run_gemm<T, true, true>(M, fout, fin, Ain, fin, 0, W, fin, 0, 1, epi, st, split_ws, P.split_floats);
+        };
         if (l < L - 1) {
             T* Aout = reinterpret_cast<T*>(ws + P.off_act[l + 1]);
-            e = run_gemm<T, true, true>(M, fout, fin, Ain, fin, 0, W, fin, 0, 1, EpiHidden<T>{bias, Aout, fout}, st,
-                                        split_ws, P.split_floats);
+            e = fwd(EpiHidden<T>{bias, Aout, fout});
             Ain = Aout;
         } else {
-            e = run_gemm<T, true, true>(M, fout, fin, Ain, fin, 0, W, fin, 0, 1, EpiLogits{bias, logits, fout}, st,
-                                        split_ws, P.split_floats);
+            e = fwd(EpiLogits{bias, logits, fout});
         }
         if (e != cudaSuccess) return fail(DBW_ECUDA, "forward GEMM %d: %s", l, cudaGetErrorString(e));
     }
@@ -457,6 +507,20 @@ bool make_grads_plan(int L, const int32_t* widths, int n, int B, int prec, Grads
     }
     P->split_floats = split;
     P->off_split = split ? take(split * 4) : 0;
+    // forward GEMMs with at least 2^27 multiply-adds and 32 outputs run in three tf32 passes
+    size_t a_parts = 0, w_parts = 0;
+    for (int l = 0; l < L; ++l) {
+        const int fin = widths[l], fout = widths[l + 1];
+        P->tf32[l] = prec == DBW_PREC_FP32 && fout >= 32 && (int64_t)P->M * fout * fin >= (int64_t(1) << 27);
+        if (!P->tf32[l]) continue;
+        const size_t ld4 = (size_t)(fin + 3) / 4 * 4;
+        a_parts = (size_t)P->M * ld4 > a_parts ? (size_t)P->M * ld4 : a_parts;
+        w_parts = (size_t)fout * ld4 > w_parts ? (size_t)fout * ld4 : w_parts;
+    }
+    P->off_ahi = a_parts ? take(a_parts * 4) : 0;
+    P->off_alo = a_parts ? take(a_parts * 4) : 0;
+    P->off_whi = w_parts ? take(w_parts * 4) : 0;
+    P->off_wlo = w_parts ? take(w_parts * 4) : 0;
     P->ws_bytes = cur;
     return true;
 }

@@ -24,6 +24,11 @@ struct GradsPlan {
     size_t off_wb;                  // bf16 weights [d] (bf16 only)
     size_t off_split;               // split-K partial tiles of the SIMT GEMMs
     size_t split_floats;
+    // fp32 forward GEMMs on the tensor cores in three tf32 passes (gemm_tf32.cuh):
+    // tf32[l] says layer l's forward GEMM takes that path; its operands' hi / lo parts
+    // go to off_ahi / off_alo ([M, ceil4(in)]) and off_whi / off_wlo ([out, ceil4(in)])
+    bool tf32[DBW_LMAX];
+    size_t off_ahi, off_alo, off_whi, off_wlo;
     size_t ws_bytes;
 };
 

@@ -191,8 +191,7 @@ class Iteration:
 
     def launches_per_step(self):
         """Kernels libdbw launches per step (for the bench's launch count); the status-word
-        memsets are copies, not kernels.  On the fp32 SIMT path a split-K GEMM adds one
-        reduce kernel, which this count leaves out."""
+        memsets are copies, not kernels."""
         L = len(self.wl.widths) - 1
         choose = (0 if self.static_b is not None else 1) + (3 if self.clock == "psw" else 0)   # + arrivals, record, fit
         # loss + dZ (+ dZ^T, written by the same kernel when its transposing tile fits)
@@ -211,7 +210,34 @@ class Iteration:
             grads = 1 + L + 1 + L + L + (L - 1)    # gather, forward, loss, dW, bias, dX
             if self.wl.prec == dbw.PREC_BF16:
                 grads += 1                          # bf16 weight cast
+            grads += self._simt_extra_launches()
         return choose + grads + 1 + 1 + 2
+
+    def _simt_extra_launches(self):
+        """Launches beyond one per GEMM on the SIMT pass: a forward GEMM in three tf32
+        passes splits its two operands first (2), a split-K GEMM sums its splits (1).
+        Mirrors the plan's rules in csrc/grads.cu."""
+        wd, M = self.wl.widths, self.wl.n * self.wl.B
+        sms = torch.cuda.get_device_properties(self.device).multi_processor_count
+
+        def split_launch(m, n, k):
+            tiles = -(-n // 128) * -(-m // 128)
+            s = min(-(-2 * sms // tiles), k // 64)
+            if s <= 1:
+                return 0
+            kps = -(-(-(-k // s)) // 16) * 16
+            return 1 if -(-k // kps) > 1 else 0
+
+        extra = 0
+        for l in range(len(wd) - 1):
+            fin, fout = wd[l], wd[l + 1]
+            if self.wl.prec == dbw.PREC_FP32 and fout >= 32 and M * fout * fin >= 1 << 27:
+                extra += 2
+            else:
+                extra += split_launch(M, fout, fin)
+            if l > 0:
+                extra += split_launch(M, fin, fout)
+        return extra
 
 
 def agg_case(n, d, seed, b, device="cuda", mean=0.0, std=1.0):

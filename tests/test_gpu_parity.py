@@ -368,6 +368,15 @@ WIDE_BF16 = workloads.Workload(
 SMALL_FP32_RAGGED = workloads.Workload(
     key="small_fp32", widths=(132, 200, 70, 7), n=5, B=3, prec=workloads.PREC_FP32, S=50,
     feature_dist="uniform", time_model="pareto", time_params={"alpha": 2.0, "xm": 1.0}, lr=0.05, seed_offset=78)
+# fp32 forward GEMMs of at least 2^27 multiply-adds run in three tf32 passes on the tensor
+# cores: M = 11 x 131 = 1441 rows (a partial 128-row tile); layer 1 with K = 1028 (a partial
+# 32-deep K block) and 322 outputs (a partial 64-column tile); layer 2, its input from the
+# first, with K = 322 (operand rows padded to 324 floats) and 330 outputs; the logits
+# layer stays on SIMT
+TF32_RAGGED = workloads.Workload(
+    key="tf32_ragged", widths=(1028, 322, 330, 5), n=11, B=131, prec=workloads.PREC_FP32, S=3000,
+    feature_dist="normal", time_model="lognormal", time_params={"mu": 0.0, "sigma": 0.5}, lr=0.01,
+    seed_offset=83)
 
 
 def grads_case(wl, t=0):
@@ -380,7 +389,7 @@ def grads_case(wl, t=0):
     return it, idx
 
 
-@pytest.mark.parametrize("wl", [workloads.SOFTMAX784, workloads.MLP784, SMALL_FP32_RAGGED, SMALL_BF16,
+@pytest.mark.parametrize("wl", [workloads.SOFTMAX784, workloads.MLP784, SMALL_FP32_RAGGED, TF32_RAGGED, SMALL_BF16,
                                 SMALL_BF16_SIMT, ODD_BF16, UNALIGNED_BF16, WIDE_BF16], ids=lambda w: w.key)
 def test_worker_grads_parity_full(wl):
     it, idx = grads_case(wl)
