@@ -48,10 +48,33 @@ struct Operands {
     CUtensorMap a_hi, a_lo, b_hi, b_lo;   // A [M, K], B [N, K], fp32 row-major, K contiguous
 };
 
+// x rounded to the nearest tf32 value (10 mantissa bits; ties to even), for finite x; a
+// value that would round up past the largest finite float is truncated instead.
+__device__ __forceinline__ float round_tf32(float x) {
+    const uint32_t u = __float_as_uint(x);
+    const uint32_t r = (u + 0x0FFFu + ((u >> 13) & 1u)) & 0xFFFFE000u;
+    return ((r & 0x7F800000u) == 0x7F800000u) ? __uint_as_float(u & 0xFFFFE000u) : __uint_as_float(r);
+}
+// hi = x rounded to nearest tf32, lo = x - hi (exact) rounded to nearest tf32.  A value
+// that is not finite goes whole to hi (a NaN as the canonical quiet NaN), lo = 0.
+__device__ __forceinline__ void split_value(float x, float& hi, float& lo) {
+    if (isfinite(x)) {
+        hi = round_tf32(x);
+        lo = round_tf32(x - hi);
+    } else {
+        hi = isnan(x) ? __uint_as_float(0x7FC00000u) : x;
+        lo = 0.f;
+    }
+}
+
 // hi / lo parts of a row-major fp32 matrix [rows, cols] (row stride lds) into two
 // matrices with row stride ldo.
 __global__ void split_kernel(const float* __restrict__ src, int rows, int cols, int64_t lds,
                              float* __restrict__ hi, float* __restrict__ lo, int64_t ldo);
+// The same, transposed: hiT[c * ldt + r], loT[c * ldt + r] for r < rows, c < cols
+// (32 x 32 tiles through shared memory; blocks of 32 x 8 threads).
+__global__ void split_t_kernel(const float* __restrict__ src, int rows, int cols, int64_t lds,
+                               float* __restrict__ hiT, float* __restrict__ loT, int64_t ldt);
 
 template <int BN, int STAGES, int NMAIN, class Epi>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -219,6 +242,248 @@ cudaError_t run(int M, int N, int K, const float* A, int64_t lda, const float* B
     if (e != cudaSuccess) return e;
     dim3 grid((N + kBN - 1) / kBN, (M + BM - 1) / BM);
     kern<<<grid, kThreads, C::SMEM, st>>>(op, M, N, K, epi, status);
+    return cudaGetLastError();
+}
+
+
+// ------------------------------------------------------------------ per-worker weight gradient
+// G[z, off + o ldrow + c] = sum_{r < K} dZ[z K + r, o] act[z K + r, c] for every worker z,
+// in three tf32 passes: A = the hi / lo parts of dZ^T [Mr = out rows, z K + r], B = those
+// of act^T [Nr = in rows, z K + r], both K-major (the transposed parts are written by
+// split_t_kernel).  A persistent grid walks 128 x 128 tiles (out x in) worker-major with
+// the in-tiles fastest; each tile has a hi.hi accumulator and a correction accumulator
+// (256 TMEM columns), two tiles in flight (512 columns), so that the MMAs of tile i + 1
+// run while the epilogue drains tile i.  With K = B <= 256 the hi.hi accumulator takes at
+// most 32 MMA additions.  Four epilogue warps, one per TMEM lane quarter (32 G rows),
+// each copy their 32 x 128 block TMEM -> registers (hi.hi + corrections, rounded to
+// nearest) -> shared memory (16-byte pieces XOR-swizzled by row) and then store it row by
+// row, 512 contiguous bytes of one G row per instruction.
+namespace dw {
+constexpr int BN = 128;
+constexpr int STAGES = 2;
+constexpr int EPI_WARPS = 4;
+constexpr int THREADS = 32 * (2 + EPI_WARPS);
+constexpr int A_BYTES = BM * BK * 4;
+constexpr int B_BYTES = BN * BK * 4;
+constexpr int STAGE_BYTES = 2 * A_BYTES + 2 * B_BYTES;   // A_hi, A_lo, B_hi, B_lo
+constexpr int WARP_STAGING = 32 * BN * 4;                // 32 rows x 512 bytes
+constexpr int SMEM = STAGES * STAGE_BYTES + EPI_WARPS * WARP_STAGING + 256 + 1024;
+constexpr int TILE_COLS = 2 * BN;                         // hi.hi, then the corrections
+constexpr int TMEM_COLS = 2 * TILE_COLS;
+constexpr int kMaxK = 256;
+}  // namespace dw
+
+static __global__ void __launch_bounds__(dw::THREADS, 1)
+    dw_kernel(const __grid_constant__ Operands op, int Mr, int Nr, int K, int batch, int* status,
+              float* __restrict__ Gbase, int64_t ldrow, int64_t ldG) {
+    using namespace tcx;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    auto part = [&](int s, int which) {
+        const int off = which < 2 ? which * dw::A_BYTES : 2 * dw::A_BYTES + (which - 2) * dw::B_BYTES;
+        return smem + s * dw::STAGE_BYTES + off;
+    };
+    uint8_t* staging = smem + dw::STAGES * dw::STAGE_BYTES;
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(staging + dw::EPI_WARPS * dw::WARP_STAGING);
+    uint64_t* empty_bar = full_bar + dw::STAGES;
+    uint64_t* tfull_bar = empty_bar + dw::STAGES;   // [2] accumulator ready
+    uint64_t* tempty_bar = tfull_bar + 2;           // [2] accumulator drained (every epilogue warp)
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty_bar + 2);
+    int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int mt_n = (Mr + BM - 1) / BM, nt_n = (Nr + dw::BN - 1) / dw::BN;
+    const int tiles_per_z = mt_n * nt_n;
+    const long long total = static_cast<long long>(tiles_per_z) * batch;
+    const int nk = (K + BK - 1) / BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < dw::STAGES; ++s) {
+            mbar_init(smem_u32(full_bar + s), 1);
+            mbar_init(smem_u32(empty_bar + s), 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(smem_u32(tfull_bar + a), 1);
+            mbar_init(smem_u32(tempty_bar + a), dw::EPI_WARPS);
+        }
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tc_alloc(smem_u32(tmem_slot), dw::TMEM_COLS);
+        tc_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    volatile int* vabort = abort_flag;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer
+        long long g = 0, issued = 0;
+        for (long long t = blockIdx.x; t < total && !*vabort; t += gridDim.x) {
+            const int z = static_cast<int>(t / tiles_per_z);
+            const int rem = static_cast<int>(t % tiles_per_z);
+            const int m0 = (rem / nt_n) * BM, n0 = (rem % nt_n) * dw::BN;
+            for (int kb = 0; kb < nk; ++kb, ++g) {
+                const int s = static_cast<int>(g % dw::STAGES);
+                const uint32_t ph = static_cast<uint32_t>((g / dw::STAGES) & 1);
+                if (!mbar_wait(smem_u32(empty_bar + s), ph ^ 1)) {
+                    atomicOr(status, 1);
+                    *vabort = 1;
+                    break;
+                }
+                const uint32_t fb = smem_u32(full_bar + s);
+                mbar_expect_tx(fb, dw::STAGE_BYTES);
+                const int kx = z * K + kb * BK;
+                tma_load_2d(smem_u32(part(s, 0)), &op.a_hi, kx, m0, fb);
+                tma_load_2d(smem_u32(part(s, 1)), &op.a_lo, kx, m0, fb);
+                tma_load_2d(smem_u32(part(s, 2)), &op.b_hi, kx, n0, fb);
+                tma_load_2d(smem_u32(part(s, 3)), &op.b_lo, kx, n0, fb);
+                issued = g + 1;
+            }
+        }
+        if (*vabort) {
+            for (long long q = issued - dw::STAGES < 0 ? 0 : issued - dw::STAGES; q < issued; ++q)
+                mbar_wait(smem_u32(full_bar + q % dw::STAGES), static_cast<uint32_t>((q / dw::STAGES) & 1));
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer
+        constexpr uint32_t idesc = instr_desc_tf32(BM, dw::BN);
+        long long g = 0;
+        int i = 0;
+        for (long long t = blockIdx.x; t < total && !*vabort; t += gridDim.x, ++i) {
+            const int acc = i & 1;
+            const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
+            if (!mbar_wait(smem_u32(tempty_bar + acc), aph ^ 1)) {
+                atomicOr(status, 1);
+                *vabort = 1;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t dmain = tmem + static_cast<uint32_t>(acc * dw::TILE_COLS);
+            const uint32_t dcorr = dmain + dw::BN;
+            bool ok = true;
+            for (int kb = 0; kb < nk; ++kb, ++g) {
+                const int s = static_cast<int>(g % dw::STAGES);
+                const uint32_t ph = static_cast<uint32_t>((g / dw::STAGES) & 1);
+                if (!mbar_wait(smem_u32(full_bar + s), ph)) {
+                    atomicOr(status, 1);
+                    *vabort = 1;
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t ah = smem_u32(part(s, 0)), al = smem_u32(part(s, 1));
+                const uint32_t bh = smem_u32(part(s, 2)), bl = smem_u32(part(s, 3));
+#pragma unroll
+                for (int kk = 0; kk < BK / 8; ++kk) {
+                    const uint32_t o = kk * 32;
+                    const uint32_t accum = (kb > 0 || kk > 0) ? 1u : 0u;
+                    tc_mma_tf32(dmain, smem_desc(ah + o, 128), smem_desc(bh + o, 128), idesc, accum);
+                    tc_mma_tf32(dcorr, smem_desc(ah + o, 128), smem_desc(bl + o, 128), idesc, accum);
+                    tc_mma_tf32(dcorr, smem_desc(al + o, 128), smem_desc(bh + o, 128), idesc, 1u);
+                }
+                tc_commit(smem_u32(empty_bar + s));
+            }
+            tc_commit(smem_u32(tfull_bar + acc));
+            if (!ok) break;
+        }
+    } else if (warp >= 2) {
+        // ---------------- epilogue
+        const int q = warp & 3;   // TMEM lanes 32 q .. 32 q + 31 = G rows m0 + 32 q ..
+        uint8_t* buf = staging + (warp - 2) * dw::WARP_STAGING;
+        int i = 0;
+        for (long long t = blockIdx.x; t < total; t += gridDim.x, ++i) {
+            const int acc = i & 1;
+            const uint32_t aph = static_cast<uint32_t>((i >> 1) & 1);
+            if (!mbar_wait(smem_u32(tfull_bar + acc), aph)) {
+                atomicOr(status, 1);
+                *vabort = 1;
+                break;
+            }
+            if (*vabort) break;
+            tc_fence_after();
+            const int z = static_cast<int>(t / tiles_per_z);
+            const int rem = static_cast<int>(t % tiles_per_z);
+            const int m0 = (rem / nt_n) * BM, n0 = (rem % nt_n) * dw::BN;
+            const uint32_t tbase =
+                tmem + static_cast<uint32_t>(acc * dw::TILE_COLS) + (static_cast<uint32_t>(q * 32) << 16);
+            const int row0 = m0 + q * 32;
+            if (row0 < Mr) {
+                // TMEM -> smem: lane = row; piece p of 128-byte segment sgm of row r at
+                // r * 512 + sgm * 128 + ((p ^ (r & 7)) * 16)
+#pragma unroll 1
+                for (int sgm = 0; sgm < dw::BN / 32; ++sgm) {
+                    uint32_t rm[32], rc[32];
+                    tc_ld_32cols(tbase + sgm * 32, rm);
+                    tc_ld_32cols(tbase + dw::BN + sgm * 32, rc);
+                    tc_wait_ld();
+#pragma unroll
+                    for (int pc = 0; pc < 8; ++pc) {
+                        float4 v;
+                        v.x = u2f(rm[4 * pc]) + u2f(rc[4 * pc]);
+                        v.y = u2f(rm[4 * pc + 1]) + u2f(rc[4 * pc + 1]);
+                        v.z = u2f(rm[4 * pc + 2]) + u2f(rc[4 * pc + 2]);
+                        v.w = u2f(rm[4 * pc + 3]) + u2f(rc[4 * pc + 3]);
+                        *reinterpret_cast<float4*>(buf + lane * 512 + sgm * 128 + ((pc ^ (lane & 7)) << 4)) = v;
+                    }
+                }
+                __syncwarp();
+                // smem -> G, one row per instruction: lane L writes columns n0 + 4 L .. + 3
+                const int sgm = lane >> 3, pc = lane & 7;
+                const int col = n0 + 4 * lane;
+                const bool col_ok = col + 3 < Nr;   // Nr % 4 == 0: whole pieces in or out
+                float* gcol = Gbase + static_cast<int64_t>(z) * ldG + col;
+#pragma unroll 4
+                for (int rr = 0; rr < 32; ++rr) {
+                    const float4 v =
+                        *reinterpret_cast<const float4*>(buf + rr * 512 + sgm * 128 + ((pc ^ (rr & 7)) << 4));
+                    if (col_ok && row0 + rr < Mr)
+                        __stcs(reinterpret_cast<float4*>(gcol + static_cast<int64_t>(row0 + rr) * ldrow), v);
+                }
+                __syncwarp();
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(tempty_bar + acc));
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tc_dealloc(tmem, dw::TMEM_COLS);
+    }
+}
+
+// Per-worker weight gradient of one layer: dz [batch K, Mr] and act [batch K, Nr]
+// (row-major fp32, row strides ldz / lda) -> G[z ldG + o ldrow + c] (Gbase = G + the
+// layer's offset).  Needs K % 32 == 0, K <= 256, Nr % 4 == 0, ldrow % 4 == 0, ldG % 4 == 0
+// and Gbase 16-byte aligned (the caller checks).  zt_hi / zt_lo: [Mr, batch K] scratch,
+// at_hi / at_lo: [Nr, batch K] scratch.
+inline cudaError_t run_dw(int Mr, int Nr, int K, int batch, const float* dz, int64_t ldz, const float* act,
+                          int64_t lda, float* zt_hi, float* zt_lo, float* at_hi, float* at_lo, float* Gbase,
+                          int64_t ldrow, int64_t ldG, int* status, cudaStream_t st) {
+    const int64_t Mt = static_cast<int64_t>(batch) * K;   // rows of dz / act = columns of the transposes
+    const dim3 blk(32, 8);
+    {
+        const int64_t ry = (Mt + 31) / 32;
+        dim3 g((Mr + 31) / 32, ry < 65535 ? static_cast<unsigned>(ry) : 65535u);
+        split_t_kernel<<<g, blk, 0, st>>>(dz, static_cast<int>(Mt), Mr, ldz, zt_hi, zt_lo, Mt);
+        dim3 g2((Nr + 31) / 32, g.y);
+        split_t_kernel<<<g2, blk, 0, st>>>(act, static_cast<int>(Mt), Nr, lda, at_hi, at_lo, Mt);
+    }
+    Operands op;
+    if (!tc_make_map_f32(&op.a_hi, zt_hi, Mr, Mt, Mt, BM) || !tc_make_map_f32(&op.a_lo, zt_lo, Mr, Mt, Mt, BM) ||
+        !tc_make_map_f32(&op.b_hi, at_hi, Nr, Mt, Mt, dw::BN) || !tc_make_map_f32(&op.b_lo, at_lo, Nr, Mt, Mt, dw::BN))
+        return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(dw_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, dw::SMEM);
+    if (e != cudaSuccess) return e;
+    const long long tiles = static_cast<long long>((Mr + BM - 1) / BM) * ((Nr + dw::BN - 1) / dw::BN) * batch;
+    const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
+    dw_kernel<<<grid, dw::THREADS, dw::SMEM, st>>>(op, Mr, Nr, K, batch, status, Gbase, ldrow, ldG);
     return cudaGetLastError();
 }
 

@@ -25,33 +25,42 @@
 namespace dbw {
 
 namespace tf32 {
-// x rounded to the nearest tf32 value (10 mantissa bits; ties to even), for finite x; a
-// value that would round up past the largest finite float is truncated instead.
-__device__ __forceinline__ float round_tf32(float x) {
-    const uint32_t u = __float_as_uint(x);
-    const uint32_t r = (u + 0x0FFFu + ((u >> 13) & 1u)) & 0xFFFFE000u;
-    return ((r & 0x7F800000u) == 0x7F800000u) ? __uint_as_float(u & 0xFFFFE000u) : __uint_as_float(r);
-}
-
-// hi = x rounded to nearest tf32, lo = x - hi (exact) rounded to nearest tf32.  A value
-// that is not finite goes whole to hi (a NaN as the canonical quiet NaN), lo = 0.
 __global__ void split_kernel(const float* __restrict__ src, int rows, int cols, int64_t lds, float* __restrict__ hi,
                              float* __restrict__ lo, int64_t ldo) {
     for (int r = blockIdx.y; r < rows; r += gridDim.y) {
         const float* s = src + (int64_t)r * lds;
         for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < cols; c += gridDim.x * blockDim.x) {
-            const float x = s[c];
             float h, l;
-            if (isfinite(x)) {
-                h = round_tf32(x);
-                l = round_tf32(x - h);
-            } else {
-                h = isnan(x) ? __uint_as_float(0x7FC00000u) : x;
-                l = 0.f;
-            }
+            split_value(s[c], h, l);
             hi[(int64_t)r * ldo + c] = h;
             lo[(int64_t)r * ldo + c] = l;
         }
+    }
+}
+
+__global__ void split_t_kernel(const float* __restrict__ src, int rows, int cols, int64_t lds,
+                               float* __restrict__ hiT, float* __restrict__ loT, int64_t ldt) {
+    __shared__ float tile[32][33];
+    const int tx = threadIdx.x, ty = threadIdx.y;
+    const int c0 = blockIdx.x * 32;
+    for (int64_t r0 = (int64_t)blockIdx.y * 32; r0 < rows; r0 += (int64_t)gridDim.y * 32) {
+        for (int j = ty; j < 32; j += 8) {
+            const int64_t r = r0 + j;
+            const int c = c0 + tx;
+            tile[j][tx] = (r < rows && c < cols) ? src[r * lds + c] : 0.f;
+        }
+        __syncthreads();
+        for (int j = ty; j < 32; j += 8) {
+            const int c = c0 + j;
+            const int64_t r = r0 + tx;
+            if (c < cols && r < rows) {
+                float h, l;
+                split_value(tile[tx][j], h, l);
+                hiT[(int64_t)c * ldt + r] = h;
+                loT[(int64_t)c * ldt + r] = l;
+            }
+        }
+        __syncthreads();
     }
 }
 }  // namespace tf32
@@ -276,6 +285,8 @@ __global__ void __launch_bounds__(256) softmax_xent_kernel(const float* __restri
                                                            float* __restrict__ loss) {
     const int i = blockIdx.x;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    constexpr int kShared = 2048;   // sample losses kept in shared memory up to this B
+    __shared__ float ls[kShared];
     __shared__ int bad_s;
     if (threadIdx.x == 0) bad_s = 0;
     __syncthreads();
@@ -302,14 +313,16 @@ __global__ void __launch_bounds__(256) softmax_xent_kernel(const float* __restri
             dZ[row * C + c] = from_f<T>(bad ? NAN : g * invB);
         }
         if (lane == 0) {
-            sample_loss[row] = bad ? NAN : (mx + logf(se)) - z[y];
+            const float l = bad ? NAN : (mx + logf(se)) - z[y];
+            sample_loss[row] = l;
+            if (r < kShared) ls[r] = l;
             if (bad) bad_s = 1;
         }
     }
     __syncthreads();
     if (threadIdx.x == 0) {
         float acc = 0.f;
-        for (int r = 0; r < B; ++r) acc += sample_loss[(int64_t)i * B + r];
+        for (int r = 0; r < B; ++r) acc += r < kShared ? ls[r] : sample_loss[(int64_t)i * B + r];
         loss[i] = bad_s ? NAN : acc * invB;
     }
 }
@@ -338,6 +351,71 @@ int splitk_count(int M, int N, int K, int batch) {
     int s = want < most ? want : most;
     return s < 1 ? 1 : s;
 }
+
+// ------------------------------------------------------------------ skinny GEMMs
+// Forward GEMM with few outputs (the logits): C[m, n] = sum_k A[m, k] W[n, k] for
+// N <= kSkinnyN.  W sits in shared memory; one warp per row of A, lane l taking
+// k = l, l + 32, .. (coalesced) into N partial sums, which a butterfly adds across the
+// warp; lane n hands output n to the epilogue.
+constexpr int kSkinnyN = 16;
+constexpr int kSkinnyK = 32;
+constexpr size_t kSkinnySmem = 48 * 1024;
+
+template <typename T, class Epi>
+__global__ void __launch_bounds__(256) skinny_n_kernel(int M, int N, int K, const T* __restrict__ A, int64_t lda,
+                                                       const T* __restrict__ W, int64_t ldw, Epi epi) {
+    extern __shared__ float wsh[];   // W as [N, K] fp32
+    for (int e = threadIdx.x; e < N * K; e += blockDim.x) wsh[e] = to_f<T>(W[(int64_t)(e / K) * ldw + e % K]);
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    const int nwarps = (gridDim.x * blockDim.x) >> 5;
+    for (int m = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; m < M; m += nwarps) {
+        float acc[kSkinnyN];
+#pragma unroll
+        for (int n = 0; n < kSkinnyN; ++n) acc[n] = 0.f;
+        const T* a = A + (int64_t)m * lda;
+        for (int k = lane; k < K; k += 32) {
+            const float av = to_f<T>(a[k]);
+#pragma unroll
+            for (int n = 0; n < kSkinnyN; ++n)
+                if (n < N) acc[n] = fmaf(av, wsh[n * K + k], acc[n]);
+        }
+        float mine = 0.f;
+#pragma unroll
+        for (int n = 0; n < kSkinnyN; ++n) {
+            if (n < N) {
+                float v = acc[n];
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+                if (lane == n) mine = v;
+            }
+        }
+        if (lane < N) epi(0, m, lane, mine);
+    }
+}
+
+// Input-gradient GEMM with a short inner dimension (K = out <= kSkinnyK):
+// dZ_{l-1}[m, c] = (sum_{o < K} dZ_l[m, o] W[o, c]) * 1[act[m, c] > 0], the products
+// added in increasing o.  W sits in shared memory; a thread per column, rows strided
+// over blockIdx.y (the dZ_l row is a broadcast load).
+template <typename T>
+__global__ void __launch_bounds__(256) skinny_k_dx_kernel(int M, int N, int K, const T* __restrict__ dZ, int64_t ldz,
+                                                          const T* __restrict__ W, int64_t ldw, EpiDx<T> epi) {
+    extern __shared__ float wsh[];   // W as [K, N] fp32
+    for (int e = threadIdx.x; e < N * K; e += blockDim.x) wsh[e] = to_f<T>(W[(int64_t)(e / N) * ldw + e % N]);
+    __syncthreads();
+    for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < N; c += gridDim.x * blockDim.x) {
+        for (int m = blockIdx.y; m < M; m += gridDim.y) {
+            const T* z = dZ + (int64_t)m * ldz;
+            float v = 0.f;
+            for (int o = 0; o < K; ++o) v = fmaf(to_f<T>(z[o]), wsh[o * N + c], v);
+            epi(0, m, c, v);
+        }
+    }
+}
+
+inline bool skinny_n_ok(int N, int K) { return N <= kSkinnyN && (size_t)N * K * 4 <= kSkinnySmem; }
+inline bool skinny_k_ok(int N, int K) { return K <= kSkinnyK && (size_t)N * K * 4 <= kSkinnySmem; }
 
 template <typename T, bool A_K, bool B_K, class Epi>
 cudaError_t run_gemm(int M, int N, int K, const T* A, int64_t lda, int64_t batchA, const T* B, int64_t ldb,
@@ -412,6 +490,13 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
                     return tf32::run(M, fout, fin, Ain, fin, W, fin, part[0], part[1], part[2], part[3], epi, status,
                                      st);
             }
+            if (skinny_n_ok(fout, fin)) {
+                const int rows_per_cta = 8;
+                const int want = (M + rows_per_cta - 1) / rows_per_cta;
+                const int grid = want < 2 * sm_count() ? want : 2 * sm_count();
+                skinny_n_kernel<T><<<grid, 256, (size_t)fout * fin * 4, st>>>(M, fout, fin, Ain, fin, W, fin, epi);
+                return cudaGetLastError();
+            }
             return run_gemm<T, true, true>(M, fout, fin, Ain, fin, 0, W, fin, 0, 1, epi, st, split_ws, P.split_floats);
         };
         if (l < L - 1) {
@@ -435,8 +520,19 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
         const T* Aprev = (l == 0) ? X : reinterpret_cast<const T*>(ws + P.off_act[l]);
         const T* dZl = dz[cur];
         // per-worker weight gradient: M' = fout, N' = fin, K = B; A(o, r) = dZ[r*fout + o], B(r, c) = A[r*fin + c]
-        e = run_gemm<T, false, false>(fout, fin, B, dZl, fout, (int64_t)B * fout, Aprev, fin, (int64_t)B * fin,
-                                      P.n, EpiDW{G, ld, P.offW[l], fin}, st);
+        bool dw_done = false;
+        if constexpr (sizeof(T) == 4) {
+            if (P.tf32_dw[l]) {
+                e = tf32::run_dw(fout, fin, B, P.n, dZl, fout, Aprev, fin, reinterpret_cast<float*>(ws + P.off_zthi),
+                                 reinterpret_cast<float*>(ws + P.off_ztlo), reinterpret_cast<float*>(ws + P.off_athi),
+                                 reinterpret_cast<float*>(ws + P.off_atlo), G + P.offW[l], fin, ld,
+                                 reinterpret_cast<int*>(ws), st);
+                dw_done = true;
+            }
+        }
+        if (!dw_done)
+            e = run_gemm<T, false, false>(fout, fin, B, dZl, fout, (int64_t)B * fout, Aprev, fin, (int64_t)B * fin,
+                                          P.n, EpiDW{G, ld, P.offW[l], fin}, st);
         if (e != cudaSuccess) return fail(DBW_ECUDA, "dW GEMM %d: %s", l, cudaGetErrorString(e));
         bias_grad_kernel<T><<<dim3((fout + 127) / 128, P.n), 128, 0, st>>>(dZl, fout, B, G, ld, P.offb[l]);
         e = cudaGetLastError();
@@ -444,8 +540,16 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
         if (l > 0) {
             // dZ_{l-1}[m, c] = sum_o dZ_l[m, o] W_l[o, c]: A(m, o) = dZ[m*fout + o], B(o, c) = W[o*fin + c]
             T* dnext = dz[cur ^ 1];
-            e = run_gemm<T, true, false>(M, fin, fout, dZl, fout, 0, wop + P.offW[l], fin, 0, 1,
-                                         EpiDx<T>{Aprev, dnext, fin}, st, split_ws, P.split_floats);
+            if (skinny_k_ok(fin, fout)) {
+                dim3 grid((fin + 255) / 256, M < 4 * sm_count() ? M : 4 * sm_count());
+                skinny_k_dx_kernel<T><<<grid, 256, (size_t)fin * fout * 4, st>>>(M, fin, fout, dZl, fout,
+                                                                                  wop + P.offW[l], fin,
+                                                                                  EpiDx<T>{Aprev, dnext, fin});
+                e = cudaGetLastError();
+            } else {
+                e = run_gemm<T, true, false>(M, fin, fout, dZl, fout, 0, wop + P.offW[l], fin, 0, 1,
+                                             EpiDx<T>{Aprev, dnext, fin}, st, split_ws, P.split_floats);
+            }
             if (e != cudaSuccess) return fail(DBW_ECUDA, "dX GEMM %d: %s", l, cudaGetErrorString(e));
             cur ^= 1;
         }
@@ -521,6 +625,22 @@ bool make_grads_plan(int L, const int32_t* widths, int n, int B, int prec, Grads
     P->off_alo = a_parts ? take(a_parts * 4) : 0;
     P->off_whi = w_parts ? take(w_parts * 4) : 0;
     P->off_wlo = w_parts ? take(w_parts * 4) : 0;
+    // weight gradients with at least 2^25 multiply-adds run in three tf32 passes when each
+    // worker's samples are whole 32-deep K blocks (at most 256) and the G rows of the layer
+    // take 16-byte stores
+    size_t zt = 0, at = 0;
+    for (int l = 0; l < L; ++l) {
+        const int fin = widths[l], fout = widths[l + 1];
+        P->tf32_dw[l] = prec == DBW_PREC_FP32 && B % 32 == 0 && B <= tf32::dw::kMaxK && fin % 4 == 0 &&
+                        P->offW[l] % 4 == 0 && fout >= 32 && (int64_t)n * fout * fin * B >= (int64_t(1) << 25);
+        if (!P->tf32_dw[l]) continue;
+        zt = (size_t)fout * P->M > zt ? (size_t)fout * P->M : zt;
+        at = (size_t)fin * P->M > at ? (size_t)fin * P->M : at;
+    }
+    P->off_zthi = zt ? take(zt * 4) : 0;
+    P->off_ztlo = zt ? take(zt * 4) : 0;
+    P->off_athi = at ? take(at * 4) : 0;
+    P->off_atlo = at ? take(at * 4) : 0;
     P->ws_bytes = cur;
     return true;
 }

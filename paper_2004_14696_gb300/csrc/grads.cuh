@@ -29,6 +29,10 @@ struct GradsPlan {
     // go to off_ahi / off_alo ([M, ceil4(in)]) and off_whi / off_wlo ([out, ceil4(in)])
     bool tf32[DBW_LMAX];
     size_t off_ahi, off_alo, off_whi, off_wlo;
+    // per-worker weight gradients in three tf32 passes: tf32_dw[l]; the transposed hi / lo
+    // parts of dZ_l ([out, M]) and of the layer input ([in, M])
+    bool tf32_dw[DBW_LMAX];
+    size_t off_zthi, off_ztlo, off_athi, off_atlo;
     size_t ws_bytes;
 };
 

@@ -214,9 +214,9 @@ class Iteration:
         return choose + grads + 1 + 1 + 2
 
     def _simt_extra_launches(self):
-        """Launches beyond one per GEMM on the SIMT pass: a forward GEMM in three tf32
-        passes splits its two operands first (2), a split-K GEMM sums its splits (1).
-        Mirrors the plan's rules in csrc/grads.cu."""
+        """Launches beyond one per GEMM on the SIMT pass: a GEMM in three tf32 passes splits
+        its two operands first (2), a split-K GEMM sums its splits (1); the skinny kernels
+        are one launch.  Mirrors the plan's rules in csrc/grads.cu."""
         wd, M = self.wl.widths, self.wl.n * self.wl.B
         sms = torch.cuda.get_device_properties(self.device).multi_processor_count
 
@@ -228,14 +228,25 @@ class Iteration:
             kps = -(-(-(-k // s)) // 16) * 16
             return 1 if -(-k // kps) > 1 else 0
 
+        def skinny_n(n, k):     # the forward GEMM with few outputs
+            return n <= 16 and n * k * 4 <= 48 * 1024
+
+        def skinny_k(n, k):     # the input-gradient GEMM with a short inner dimension
+            return k <= 32 and n * k * 4 <= 48 * 1024
+
+        B, n, off = self.wl.B, self.wl.n, 0
         extra = 0
         for l in range(len(wd) - 1):
             fin, fout = wd[l], wd[l + 1]
+            if (self.wl.prec == dbw.PREC_FP32 and B % 32 == 0 and B <= 256 and fin % 4 == 0 and off % 4 == 0
+                    and fout >= 32 and n * fout * fin * B >= 1 << 25):
+                extra += 2      # the weight gradient's transposed operand parts
+            off += fin * fout + fout
             if self.wl.prec == dbw.PREC_FP32 and fout >= 32 and M * fout * fin >= 1 << 27:
                 extra += 2
-            else:
+            elif not skinny_n(fout, fin):
                 extra += split_launch(M, fout, fin)
-            if l > 0:
+            if l > 0 and not skinny_k(fin, fout):
                 extra += split_launch(M, fin, fout)
         return extra
 

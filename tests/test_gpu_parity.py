@@ -373,6 +373,13 @@ SMALL_FP32_RAGGED = workloads.Workload(
 # 32-deep K block) and 322 outputs (a partial 64-column tile); layer 2, its input from the
 # first, with K = 322 (operand rows padded to 324 floats) and 330 outputs; the logits
 # layer stays on SIMT
+# per-worker weight gradients in three tf32 passes (B = 96: three 32-deep K blocks per
+# worker): layer 1 with 200 outputs (a partial 128-row tile) and 516 inputs (a partial
+# 128-column tile of 4 columns), layer 2 on the hidden activations (G offset 103,400)
+TF32_DW = workloads.Workload(
+    key="tf32_dw", widths=(516, 200, 136, 12), n=21, B=96, prec=workloads.PREC_FP32, S=4000,
+    feature_dist="uniform", time_model="shifted_exp", time_params={"shift": 1.0, "rate": 1.0}, lr=0.01,
+    seed_offset=84)
 TF32_RAGGED = workloads.Workload(
     key="tf32_ragged", widths=(1028, 322, 330, 5), n=11, B=131, prec=workloads.PREC_FP32, S=3000,
     feature_dist="normal", time_model="lognormal", time_params={"mu": 0.0, "sigma": 0.5}, lr=0.01,
@@ -389,8 +396,9 @@ def grads_case(wl, t=0):
     return it, idx
 
 
-@pytest.mark.parametrize("wl", [workloads.SOFTMAX784, workloads.MLP784, SMALL_FP32_RAGGED, TF32_RAGGED, SMALL_BF16,
-                                SMALL_BF16_SIMT, ODD_BF16, UNALIGNED_BF16, WIDE_BF16], ids=lambda w: w.key)
+@pytest.mark.parametrize("wl", [workloads.SOFTMAX784, workloads.MLP784, SMALL_FP32_RAGGED, TF32_RAGGED, TF32_DW,
+                                SMALL_BF16, SMALL_BF16_SIMT, ODD_BF16, UNALIGNED_BF16, WIDE_BF16],
+                         ids=lambda w: w.key)
 def test_worker_grads_parity_full(wl):
     it, idx = grads_case(wl)
     pool, labels, w = it.pool.cpu().numpy(), it.labels.cpu().numpy(), it.w.cpu().numpy()
