@@ -71,6 +71,11 @@ __device__ __forceinline__ void split_value(float x, float& hi, float& lo) {
 // matrices with row stride ldo.
 __global__ void split_kernel(const float* __restrict__ src, int rows, int cols, int64_t lds,
                              float* __restrict__ hi, float* __restrict__ lo, int64_t ldo);
+// The same four values at a time (cols, lds, ldo multiples of 4; src 16-byte aligned).
+__global__ void split4_kernel(const float* __restrict__ src, int rows, int cols, int64_t lds,
+                              float* __restrict__ hi, float* __restrict__ lo, int64_t ldo);
+// Launches split4_kernel where its alignment holds, else split_kernel.
+void split(const float* src, int rows, int cols, int64_t lds, float* hi, float* lo, int64_t ldo, cudaStream_t st);
 // The same, transposed: hiT[c * ldt + r], loT[c * ldt + r] for r < rows, c < cols
 // (32 x 32 tiles through shared memory; blocks of 32 x 8 threads).
 __global__ void split_t_kernel(const float* __restrict__ src, int rows, int cols, int64_t lds,
@@ -199,11 +204,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int j = 0; j < 32; ++j) v[j] += u2f(r[j]);
                 }
-                if (row < M) {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        if (nb + j < N) epi(0, row, nb + j, v[j]);
-                }
+                if (row < M) epi.row32(row, nb, N, v);
             }
         }
     }
@@ -219,19 +220,20 @@ constexpr int kBN = 64;
 constexpr int kStages = 4;
 constexpr int kMain = 7;   // (7 + 1) x 64 = 512 TMEM columns
 
+// The epilogue functor takes a row's outputs 32 columns at a time:
+// epi.row32(m, n0, N, v) for columns n0 .. n0 + 31 (those below N).
+//
 // Splits both operands into ws buffers (a_hi, a_lo: [M, lda2]; b_hi, b_lo: [N, ldb2],
 // lda2 = ldb2 = K rounded up to 4) and runs C = A B^T into ``epi``.  A [M, K] (row
 // stride lda) and B [N, K] (row stride ldb) are fp32 row-major.
+// a_parts_ready: a_hi / a_lo already hold A's parts (written by the producer of A).
 template <class Epi>
 cudaError_t run(int M, int N, int K, const float* A, int64_t lda, const float* B, int64_t ldb, float* a_hi,
-                float* a_lo, float* b_hi, float* b_lo, Epi epi, int* status, cudaStream_t st) {
+                float* a_lo, float* b_hi, float* b_lo, Epi epi, int* status, cudaStream_t st,
+                bool a_parts_ready = false) {
     const int64_t ld2 = (K + 3) / 4 * 4;
-    {
-        dim3 g((K + 127) / 128, M < 65535 ? M : 65535);
-        split_kernel<<<g, 128, 0, st>>>(A, M, K, lda, a_hi, a_lo, ld2);
-        dim3 gb((K + 127) / 128, N < 65535 ? N : 65535);
-        split_kernel<<<gb, 128, 0, st>>>(B, N, K, ldb, b_hi, b_lo, ld2);
-    }
+    if (!a_parts_ready) split(A, M, K, lda, a_hi, a_lo, ld2, st);
+    split(B, N, K, ldb, b_hi, b_lo, ld2, st);
     Operands op;
     if (!tc_make_map_f32(&op.a_hi, a_hi, M, K, ld2, BM) || !tc_make_map_f32(&op.a_lo, a_lo, M, K, ld2, BM) ||
         !tc_make_map_f32(&op.b_hi, b_hi, N, K, ld2, kBN) || !tc_make_map_f32(&op.b_lo, b_lo, N, K, ld2, kBN))
@@ -463,17 +465,20 @@ static __global__ void __launch_bounds__(dw::THREADS, 1)
 // layer's offset).  Needs K % 32 == 0, K <= 256, Nr % 4 == 0, ldrow % 4 == 0, ldG % 4 == 0
 // and Gbase 16-byte aligned (the caller checks).  zt_hi / zt_lo: [Mr, batch K] scratch,
 // at_hi / at_lo: [Nr, batch K] scratch.
+// act_parts_ready: at_hi / at_lo already hold act's transposed parts (act is not read).
 inline cudaError_t run_dw(int Mr, int Nr, int K, int batch, const float* dz, int64_t ldz, const float* act,
                           int64_t lda, float* zt_hi, float* zt_lo, float* at_hi, float* at_lo, float* Gbase,
-                          int64_t ldrow, int64_t ldG, int* status, cudaStream_t st) {
+                          int64_t ldrow, int64_t ldG, int* status, cudaStream_t st, bool act_parts_ready = false) {
     const int64_t Mt = static_cast<int64_t>(batch) * K;   // rows of dz / act = columns of the transposes
     const dim3 blk(32, 8);
     {
         const int64_t ry = (Mt + 31) / 32;
         dim3 g((Mr + 31) / 32, ry < 65535 ? static_cast<unsigned>(ry) : 65535u);
         split_t_kernel<<<g, blk, 0, st>>>(dz, static_cast<int>(Mt), Mr, ldz, zt_hi, zt_lo, Mt);
-        dim3 g2((Nr + 31) / 32, g.y);
-        split_t_kernel<<<g2, blk, 0, st>>>(act, static_cast<int>(Mt), Nr, lda, at_hi, at_lo, Mt);
+        if (!act_parts_ready) {
+            dim3 g2((Nr + 31) / 32, g.y);
+            split_t_kernel<<<g2, blk, 0, st>>>(act, static_cast<int>(Mt), Nr, lda, at_hi, at_lo, Mt);
+        }
     }
     Operands op;
     if (!tc_make_map_f32(&op.a_hi, zt_hi, Mr, Mt, Mt, BM) || !tc_make_map_f32(&op.a_lo, zt_lo, Mr, Mt, Mt, BM) ||

@@ -38,6 +38,35 @@ __global__ void split_kernel(const float* __restrict__ src, int rows, int cols, 
     }
 }
 
+__global__ void split4_kernel(const float* __restrict__ src, int rows, int cols, int64_t lds, float* __restrict__ hi,
+                              float* __restrict__ lo, int64_t ldo) {
+    const int c4 = cols / 4;
+    const int64_t total = (int64_t)rows * c4;
+    for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < total; q += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = q / c4;
+        const int c = static_cast<int>(q - r * c4) * 4;
+        const float4 v = *reinterpret_cast<const float4*>(src + r * lds + c);
+        float4 h, l;
+        split_value(v.x, h.x, l.x);
+        split_value(v.y, h.y, l.y);
+        split_value(v.z, h.z, l.z);
+        split_value(v.w, h.w, l.w);
+        *reinterpret_cast<float4*>(hi + r * ldo + c) = h;
+        *reinterpret_cast<float4*>(lo + r * ldo + c) = l;
+    }
+}
+
+void split(const float* src, int rows, int cols, int64_t lds, float* hi, float* lo, int64_t ldo, cudaStream_t st) {
+    if (cols % 4 == 0 && lds % 4 == 0 && ldo % 4 == 0 && aligned16(src) && aligned16(hi) && aligned16(lo)) {
+        const int64_t want = ((int64_t)rows * (cols / 4) + 255) / 256;
+        const int blocks = static_cast<int>(want < 8 * sm_count() ? want : 8 * sm_count());
+        split4_kernel<<<blocks < 1 ? 1 : blocks, 256, 0, st>>>(src, rows, cols, lds, hi, lo, ldo);
+    } else {
+        dim3 g((cols + 127) / 128, rows < 65535 ? rows : 65535);
+        split_kernel<<<g, 128, 0, st>>>(src, rows, cols, lds, hi, lo, ldo);
+    }
+}
+
 __global__ void split_t_kernel(const float* __restrict__ src, int rows, int cols, int64_t lds,
                                float* __restrict__ hiT, float* __restrict__ loT, int64_t ldt) {
     __shared__ float tile[32][33];
@@ -76,10 +105,11 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float
 
 // ------------------------------------------------------------------ gather
 // X[m, :] = pool[idx[m], :].  An index outside [0, S) reads row 0; the loss
-// kernel poisons that worker.
+// kernel poisons that worker.  With hi != nullptr (fp32 pass, first forward GEMM in
+// three tf32 passes) the row's tf32 parts go to hi / lo [M, ldo] as well (ldo % 4 == 0).
 template <typename T>
 __global__ void gather_kernel(const float* __restrict__ pool, int64_t S, int in, const int32_t* __restrict__ idx,
-                              int M, T* __restrict__ X) {
+                              int M, T* __restrict__ X, float* __restrict__ hi, float* __restrict__ lo, int64_t ldo) {
     for (int m = blockIdx.y; m < M; m += gridDim.y) {
         int64_t r = idx[m];
         if (r < 0 || r >= S) r = 0;
@@ -92,9 +122,58 @@ __global__ void gather_kernel(const float* __restrict__ pool, int64_t S, int in,
                 dst[c + 1] = from_f<T>(v.y);
                 dst[c + 2] = from_f<T>(v.z);
                 dst[c + 3] = from_f<T>(v.w);
+                if (hi) {
+                    float4 h, l;
+                    tf32::split_value(v.x, h.x, l.x);
+                    tf32::split_value(v.y, h.y, l.y);
+                    tf32::split_value(v.z, h.z, l.z);
+                    tf32::split_value(v.w, h.w, l.w);
+                    *reinterpret_cast<float4*>(hi + (int64_t)m * ldo + c) = h;
+                    *reinterpret_cast<float4*>(lo + (int64_t)m * ldo + c) = l;
+                }
             } else {
-                for (int e = c; e < in; ++e) dst[e] = from_f<T>(src[e]);
+                for (int e = c; e < in; ++e) {
+                    dst[e] = from_f<T>(src[e]);
+                    if (hi) tf32::split_value(src[e], hi[(int64_t)m * ldo + e], lo[(int64_t)m * ldo + e]);
+                }
             }
+        }
+    }
+}
+
+// The gather of the fp32 pass when its first layer runs in three tf32 passes: the
+// gathered rows' tf32 parts row-major (hi / lo [M, ldo], when hi != nullptr) and
+// transposed (hiT / loT [in, ldt], when hiT != nullptr), and X itself when X != nullptr;
+// 32 x 32 tiles of X through shared memory, blocks of 32 x 8 threads.
+__global__ void gather_parts_kernel(const float* __restrict__ pool, int64_t S, int in,
+                                    const int32_t* __restrict__ idx, int M, float* __restrict__ X,
+                                    float* __restrict__ hi, float* __restrict__ lo, int64_t ldo,
+                                    float* __restrict__ hiT, float* __restrict__ loT, int64_t ldt) {
+    __shared__ float tile[32][33];
+    const int tx = threadIdx.x, ty = threadIdx.y;
+    const int c0 = blockIdx.x * 32;
+    for (int64_t m0 = (int64_t)blockIdx.y * 32; m0 < M; m0 += (int64_t)gridDim.y * 32) {
+        for (int j = ty; j < 32; j += 8) {
+            const int64_t m = m0 + j;
+            const int c = c0 + tx;
+            float v = 0.f;
+            if (m < M && c < in) {
+                int64_t r = idx[m];
+                if (r < 0 || r >= S) r = 0;
+                v = pool[r * in + c];
+                if (X) X[m * in + c] = v;
+                if (hi) tf32::split_value(v, hi[m * ldo + c], lo[m * ldo + c]);
+            }
+            tile[j][tx] = v;
+        }
+        if (hiT) {
+            __syncthreads();
+            for (int j = ty; j < 32; j += 8) {
+                const int c = c0 + j;
+                const int64_t m = m0 + tx;
+                if (c < in && m < M) tf32::split_value(tile[tx][j], hiT[(int64_t)c * ldt + m], loT[(int64_t)c * ldt + m]);
+            }
+            __syncthreads();
         }
     }
 }
@@ -240,6 +319,18 @@ struct EpiHidden {
         v += bias[n];
         out[(int64_t)m * ldo + n] = from_f<T>(v > 0.f ? v : 0.f);
     }
+    // 32 consecutive outputs of row m from column n0 (those below N): the biases are
+    // loaded before any store
+    __device__ __forceinline__ void row32(int m, int n0, int N, const float (&v)[32]) const {
+        float b[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) b[j] = n0 + j < N ? bias[n0 + j] : 0.f;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            const float x = v[j] + b[j];
+            if (n0 + j < N) out[(int64_t)m * ldo + n0 + j] = from_f<T>(x > 0.f ? x : 0.f);
+        }
+    }
 };
 // forward last layer: logits = C + b (fp32)
 struct EpiLogits {
@@ -248,6 +339,14 @@ struct EpiLogits {
     int ldo;
     __device__ __forceinline__ void operator()(int, int m, int n, float v) const {
         out[(int64_t)m * ldo + n] = v + bias[n];
+    }
+    __device__ __forceinline__ void row32(int m, int n0, int N, const float (&v)[32]) const {
+        float b[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) b[j] = n0 + j < N ? bias[n0 + j] : 0.f;
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (n0 + j < N) out[(int64_t)m * ldo + n0 + j] = v[j] + b[j];
     }
 };
 // input gradient: dZ_{l-1} = C * 1[A_{l-1} > 0]  (a product, so a NaN-poisoned row stays NaN)
@@ -291,7 +390,55 @@ __global__ void __launch_bounds__(256) softmax_xent_kernel(const float* __restri
     if (threadIdx.x == 0) bad_s = 0;
     __syncthreads();
     const float invB = 1.0f / (float)B;
-    for (int r = warp; r < B; r += nw) {
+    if (C <= 32) {
+        // lane c holds class c; a warp's rows go in batches of 8 whose logits, sample
+        // indices and labels are all loaded before the first is reduced
+        for (int r0 = warp; r0 < B; r0 += 8 * nw) {
+            float zv[8];
+            int yv[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int r = r0 + j * nw;
+                zv[j] = -INFINITY;
+                yv[j] = -1;
+                if (r < B) {
+                    const int64_t row = (int64_t)i * B + r;
+                    if (lane < C) zv[j] = logits[row * C + lane];
+                    const int64_t sidx = idx[row];
+                    if (sidx >= 0 && sidx < S) yv[j] = labels[sidx];
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int r = r0 + j * nw;
+                if (r >= B) break;
+                const int64_t row = (int64_t)i * B + r;
+                const int y = yv[j];
+                const bool bad = (y < 0 || y >= C);
+                float mx = zv[j];
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+                const float ex = lane < C ? expf(zv[j] - mx) : 0.f;
+                float se = ex;
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
+                const float inv_se = 1.0f / se;
+                if (lane < C) {
+                    float g = ex * inv_se;
+                    if (lane == y) g -= 1.0f;
+                    dZ[row * C + lane] = from_f<T>(bad ? NAN : g * invB);
+                }
+                const float zy = __shfl_sync(0xffffffffu, zv[j], bad ? 0 : y);
+                if (lane == 0) {
+                    const float l = bad ? NAN : (mx + logf(se)) - zy;
+                    sample_loss[row] = l;
+                    if (r < kShared) ls[r] = l;
+                    if (bad) bad_s = 1;
+                }
+            }
+        }
+    }
+    for (int r = C <= 32 ? B : warp; r < B; r += nw) {
         const int64_t row = (int64_t)i * B + r;
         const int64_t sidx = idx[row];
         int y = -1;
@@ -337,6 +484,7 @@ __global__ void bias_grad_kernel(const T* __restrict__ dZ, int out, int B, float
     if (o >= out) return;
     const T* p = dZ + (int64_t)i * B * out + o;
     float acc = 0.f;
+#pragma unroll 16
     for (int r = 0; r < B; ++r) acc += to_f<T>(p[(int64_t)r * out]);
     G[(int64_t)i * ldG + offb + o] = acc;
 }
@@ -352,6 +500,25 @@ int splitk_count(int M, int N, int K, int batch) {
     return s < 1 ? 1 : s;
 }
 
+// Fills dst[e] = f(e) for e < count, each thread loading 8 values before storing any
+// (so that one thread's loads are in flight together, not one per store).
+template <class F>
+__device__ __forceinline__ void fill_shared(float* dst, int count, F f) {
+    for (int e0 = threadIdx.x; e0 < count; e0 += 8 * blockDim.x) {
+        float t[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int e = e0 + u * blockDim.x;
+            t[u] = e < count ? f(e) : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int e = e0 + u * blockDim.x;
+            if (e < count) dst[e] = t[u];
+        }
+    }
+}
+
 // ------------------------------------------------------------------ skinny GEMMs
 // Forward GEMM with few outputs (the logits): C[m, n] = sum_k A[m, k] W[n, k] for
 // N <= kSkinnyN.  W sits in shared memory; one warp per row of A, lane l taking
@@ -365,7 +532,7 @@ template <typename T, class Epi>
 __global__ void __launch_bounds__(256) skinny_n_kernel(int M, int N, int K, const T* __restrict__ A, int64_t lda,
                                                        const T* __restrict__ W, int64_t ldw, Epi epi) {
     extern __shared__ float wsh[];   // W as [N, K] fp32
-    for (int e = threadIdx.x; e < N * K; e += blockDim.x) wsh[e] = to_f<T>(W[(int64_t)(e / K) * ldw + e % K]);
+    fill_shared(wsh, N * K, [&](int e) { return to_f<T>(W[(int64_t)(e / K) * ldw + e % K]); });
     __syncthreads();
     const int lane = threadIdx.x & 31;
     const int nwarps = (gridDim.x * blockDim.x) >> 5;
@@ -374,11 +541,20 @@ __global__ void __launch_bounds__(256) skinny_n_kernel(int M, int N, int K, cons
 #pragma unroll
         for (int n = 0; n < kSkinnyN; ++n) acc[n] = 0.f;
         const T* a = A + (int64_t)m * lda;
-        for (int k = lane; k < K; k += 32) {
-            const float av = to_f<T>(a[k]);
+        // 8 of the lane's elements loaded at a time, then multiplied
+        for (int k0 = lane; k0 < K; k0 += 8 * 32) {
+            float av[8];
 #pragma unroll
-            for (int n = 0; n < kSkinnyN; ++n)
-                if (n < N) acc[n] = fmaf(av, wsh[n * K + k], acc[n]);
+            for (int u = 0; u < 8; ++u) av[u] = k0 + 32 * u < K ? to_f<T>(a[k0 + 32 * u]) : 0.f;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int k = k0 + 32 * u;
+                if (k < K) {
+#pragma unroll
+                    for (int n = 0; n < kSkinnyN; ++n)
+                        if (n < N) acc[n] = fmaf(av[u], wsh[n * K + k], acc[n]);
+                }
+            }
         }
         float mine = 0.f;
 #pragma unroll
@@ -396,26 +572,45 @@ __global__ void __launch_bounds__(256) skinny_n_kernel(int M, int N, int K, cons
 
 // Input-gradient GEMM with a short inner dimension (K = out <= kSkinnyK):
 // dZ_{l-1}[m, c] = (sum_{o < K} dZ_l[m, o] W[o, c]) * 1[act[m, c] > 0], the products
-// added in increasing o.  W sits in shared memory; a thread per column, rows strided
-// over blockIdx.y (the dZ_l row is a broadcast load).
+// added in increasing o (EpiDx's arithmetic, with the 16 masks loaded before any
+// store).  W and the CTA's 16 rows of dZ_l sit in shared memory; a thread per column
+// computes the 16 rows' outputs.
 template <typename T>
 __global__ void __launch_bounds__(256) skinny_k_dx_kernel(int M, int N, int K, const T* __restrict__ dZ, int64_t ldz,
                                                           const T* __restrict__ W, int64_t ldw, EpiDx<T> epi) {
-    extern __shared__ float wsh[];   // W as [K, N] fp32
-    for (int e = threadIdx.x; e < N * K; e += blockDim.x) wsh[e] = to_f<T>(W[(int64_t)(e / N) * ldw + e % N]);
-    __syncthreads();
-    for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < N; c += gridDim.x * blockDim.x) {
-        for (int m = blockIdx.y; m < M; m += gridDim.y) {
-            const T* z = dZ + (int64_t)m * ldz;
-            float v = 0.f;
-            for (int o = 0; o < K; ++o) v = fmaf(to_f<T>(z[o]), wsh[o * N + c], v);
-            epi(0, m, c, v);
+    constexpr int R = 16;                               // rows per CTA
+    extern __shared__ float wsh[];                      // W as [K, N] fp32, then the CTA's dZ rows [R, K]
+    float* zsh = wsh + N * K;
+    fill_shared(wsh, N * K, [&](int e) { return to_f<T>(W[(int64_t)(e / N) * ldw + e % N]); });
+    for (int m0 = blockIdx.y * R; m0 < M; m0 += gridDim.y * R) {
+        __syncthreads();   // the previous rows' reads of zsh are done
+        fill_shared(zsh, R * K, [&](int e) {
+            const int m = m0 + e / K;
+            return m < M ? to_f<T>(dZ[(int64_t)m * ldz + e % K]) : 0.f;
+        });
+        __syncthreads();
+        for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < N; c += gridDim.x * blockDim.x) {
+            float v[R];
+#pragma unroll
+            for (int j = 0; j < R; ++j) v[j] = 0.f;
+            for (int o = 0; o < K; ++o) {
+                const float wv = wsh[o * N + c];
+#pragma unroll
+                for (int j = 0; j < R; ++j) v[j] = fmaf(zsh[j * K + o], wv, v[j]);
+            }
+            // the ReLU masks of the R rows, all loaded before the first store
+            float a[R];
+#pragma unroll
+            for (int j = 0; j < R; ++j) a[j] = m0 + j < M ? to_f<T>(epi.act[(int64_t)(m0 + j) * epi.ldo + c]) : 0.f;
+#pragma unroll
+            for (int j = 0; j < R; ++j)
+                if (m0 + j < M) epi.out[(int64_t)(m0 + j) * epi.ldo + c] = from_f<T>(v[j] * (a[j] > 0.f ? 1.f : 0.f));
         }
     }
 }
 
 inline bool skinny_n_ok(int N, int K) { return N <= kSkinnyN && (size_t)N * K * 4 <= kSkinnySmem; }
-inline bool skinny_k_ok(int N, int K) { return K <= kSkinnyK && (size_t)N * K * 4 <= kSkinnySmem; }
+inline bool skinny_k_ok(int N, int K) { return K <= kSkinnyK && ((size_t)N + 16) * K * 4 <= kSkinnySmem; }
 
 template <typename T, bool A_K, bool B_K, class Epi>
 cudaError_t run_gemm(int M, int N, int K, const T* A, int64_t lda, int64_t batchA, const T* B, int64_t ldb,
@@ -464,7 +659,20 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
     {
         const int in = P.widths[0];
         dim3 grid((in + 1023) / 1024, M < 65535 ? M : 65535);
-        gather_kernel<T><<<grid, 256, 0, st>>>(pool, S, in, idx, M, X);
+        if (sizeof(T) == 4 && (P.tf32[0] || P.tf32_dw[0])) {
+            // the first layer's GEMMs in three tf32 passes take their X parts from the gather;
+            // X itself only when one of them stays on SIMT
+            const int ty = (M + 31) / 32;
+            const bool need_x = !(P.tf32[0] && P.tf32_dw[0]);
+            gather_parts_kernel<<<dim3((in + 31) / 32, ty < 65535 ? ty : 65535), dim3(32, 8), 0, st>>>(
+                pool, S, in, idx, M, need_x ? reinterpret_cast<float*>(X) : nullptr,
+                P.tf32[0] ? reinterpret_cast<float*>(ws + P.off_ahi) : nullptr,
+                P.tf32[0] ? reinterpret_cast<float*>(ws + P.off_alo) : nullptr, (in + 3) / 4 * 4,
+                P.tf32_dw[0] ? reinterpret_cast<float*>(ws + P.off_xthi) : nullptr,
+                P.tf32_dw[0] ? reinterpret_cast<float*>(ws + P.off_xtlo) : nullptr, M);
+        } else {
+            gather_kernel<T><<<grid, 256, 0, st>>>(pool, S, in, idx, M, X, nullptr, nullptr, 0);
+        }
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(DBW_ECUDA, "gather launch: %s", cudaGetErrorString(e));
@@ -488,7 +696,7 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
             if constexpr (sizeof(T) == 4) {
                 if (tc)
                     return tf32::run(M, fout, fin, Ain, fin, W, fin, part[0], part[1], part[2], part[3], epi, status,
-                                     st);
+                                     st, /*a_parts_ready=*/l == 0);
             }
             if (skinny_n_ok(fout, fin)) {
                 const int rows_per_cta = 8;
@@ -523,10 +731,11 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
         bool dw_done = false;
         if constexpr (sizeof(T) == 4) {
             if (P.tf32_dw[l]) {
+                const size_t ath = l == 0 ? P.off_xthi : P.off_athi, atl = l == 0 ? P.off_xtlo : P.off_atlo;
                 e = tf32::run_dw(fout, fin, B, P.n, dZl, fout, Aprev, fin, reinterpret_cast<float*>(ws + P.off_zthi),
-                                 reinterpret_cast<float*>(ws + P.off_ztlo), reinterpret_cast<float*>(ws + P.off_athi),
-                                 reinterpret_cast<float*>(ws + P.off_atlo), G + P.offW[l], fin, ld,
-                                 reinterpret_cast<int*>(ws), st);
+                                 reinterpret_cast<float*>(ws + P.off_ztlo), reinterpret_cast<float*>(ws + ath),
+                                 reinterpret_cast<float*>(ws + atl), G + P.offW[l], fin, ld,
+                                 reinterpret_cast<int*>(ws), st, /*act_parts_ready=*/l == 0);
                 dw_done = true;
             }
         }
@@ -541,8 +750,9 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
             // dZ_{l-1}[m, c] = sum_o dZ_l[m, o] W_l[o, c]: A(m, o) = dZ[m*fout + o], B(o, c) = W[o*fin + c]
             T* dnext = dz[cur ^ 1];
             if (skinny_k_ok(fin, fout)) {
-                dim3 grid((fin + 255) / 256, M < 4 * sm_count() ? M : 4 * sm_count());
-                skinny_k_dx_kernel<T><<<grid, 256, (size_t)fin * fout * 4, st>>>(M, fin, fout, dZl, fout,
+                const int ry = (M + 15) / 16;
+                dim3 grid((fin + 255) / 256, ry < 65535 ? ry : 65535);
+                skinny_k_dx_kernel<T><<<grid, 256, ((size_t)fin + 16) * fout * 4, st>>>(M, fin, fout, dZl, fout,
                                                                                   wop + P.offW[l], fin,
                                                                                   EpiDx<T>{Aprev, dnext, fin});
                 e = cudaGetLastError();
@@ -635,12 +845,15 @@ bool make_grads_plan(int L, const int32_t* widths, int n, int B, int prec, Grads
                         P->offW[l] % 4 == 0 && fout >= 32 && (int64_t)n * fout * fin * B >= (int64_t(1) << 25);
         if (!P->tf32_dw[l]) continue;
         zt = (size_t)fout * P->M > zt ? (size_t)fout * P->M : zt;
-        at = (size_t)fin * P->M > at ? (size_t)fin * P->M : at;
+        if (l > 0) at = (size_t)fin * P->M > at ? (size_t)fin * P->M : at;
     }
     P->off_zthi = zt ? take(zt * 4) : 0;
     P->off_ztlo = zt ? take(zt * 4) : 0;
     P->off_athi = at ? take(at * 4) : 0;
     P->off_atlo = at ? take(at * 4) : 0;
+    const size_t xt = P->tf32_dw[0] ? (size_t)widths[0] * P->M : 0;
+    P->off_xthi = xt ? take(xt * 4) : 0;
+    P->off_xtlo = xt ? take(xt * 4) : 0;
     P->ws_bytes = cur;
     return true;
 }

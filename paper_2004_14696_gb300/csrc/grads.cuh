@@ -33,6 +33,7 @@ struct GradsPlan {
     // parts of dZ_l ([out, M]) and of the layer input ([in, M])
     bool tf32_dw[DBW_LMAX];
     size_t off_zthi, off_ztlo, off_athi, off_atlo;
+    size_t off_xthi, off_xtlo;      // the first layer's input parts [in, M], written by the gather
     size_t ws_bytes;
 };
 

@@ -232,7 +232,7 @@ class Iteration:
             return n <= 16 and n * k * 4 <= 48 * 1024
 
         def skinny_k(n, k):     # the input-gradient GEMM with a short inner dimension
-            return k <= 32 and n * k * 4 <= 48 * 1024
+            return k <= 32 and (n + 16) * k * 4 <= 48 * 1024
 
         B, n, off = self.wl.B, self.wl.n, 0
         extra = 0
@@ -240,10 +240,10 @@ class Iteration:
             fin, fout = wd[l], wd[l + 1]
             if (self.wl.prec == dbw.PREC_FP32 and B % 32 == 0 and B <= 256 and fin % 4 == 0 and off % 4 == 0
                     and fout >= 32 and n * fout * fin * B >= 1 << 25):
-                extra += 2      # the weight gradient's transposed operand parts
+                extra += 1 if l == 0 else 2     # transposed parts of dZ_l (and of the input above layer 1)
             off += fin * fout + fout
             if self.wl.prec == dbw.PREC_FP32 and fout >= 32 and M * fout * fin >= 1 << 27:
-                extra += 2
+                extra += 1 if l == 0 else 2     # the gather writes the first layer's input parts
             elif not skinny_n(fout, fin):
                 extra += split_launch(M, fout, fin)
             if l > 0 and not skinny_k(fin, fout):
