@@ -6,7 +6,8 @@
 // separately rounded IEEE operation, performed in the order written, so that a
 // state reproduced elsewhere with the same operation order yields the same b_t
 // bit for bit.  The sequential pieces (window sums, the loss mean) run in one
-// thread on purpose: their summation order is part of that contract.
+// thread on purpose: their summation order is part of that contract.  Their inputs
+// are first loaded into shared memory by all threads.
 #include <math.h>
 #include <math_constants.h>
 
@@ -56,10 +57,19 @@ __global__ void __launch_bounds__(1024) grad_stats_kernel(
     const float* __restrict__ loss, const double* __restrict__ tsorted, double lr,
     dbw_state* __restrict__ st, double* __restrict__ stats_out, double* __restrict__ row_sqnorm) {
     __shared__ int k_s;
+    // the mask and the losses, loaded by every thread at once; thread 0 then runs the
+    // sequential sums from shared memory (n <= DBW_NMAX: checked by the caller)
+    __shared__ uint8_t mask_s[DBW_NMAX];
+    __shared__ float loss_s[DBW_NMAX];
     const int tid = threadIdx.x;
+    for (int j = tid; j < n; j += blockDim.x) {
+        mask_s[j] = mask[j] ? 1 : 0;
+        loss_s[j] = loss[j];
+    }
+    __syncthreads();
     if (tid == 0) {
         int k = 0;
-        for (int j = 0; j < n; ++j) k += mask[j] ? 1 : 0;
+        for (int j = 0; j < n; ++j) k += mask_s[j];
         k_s = k;
         if (k == 0 || st->n != n) {
             st->flags |= (k == 0 ? DBW_FLAG_EMPTY_MASK : 0) | (st->n != n ? DBW_FLAG_BAD_STATE : 0);
@@ -72,7 +82,7 @@ __global__ void __launch_bounds__(1024) grad_stats_kernel(
         const int k = k_s;
         double acc = 0.0;
         for (int j = 0; j < n; ++j)
-            if (mask[j]) acc = acc + (double)loss[j];
+            if (mask_s[j]) acc = acc + (double)loss_s[j];
         const double SS = sums[n];
         const double g2 = sums[n + 1];
         const double F = acc / (double)k;
@@ -156,6 +166,14 @@ __global__ void __launch_bounds__(1024) choose_b_kernel(dbw_state* __restrict__ 
         return;
     }
     const bool blind = (flags & DBW_CHOOSE_BLIND) != 0;
+    // the three windows' rings, loaded by every thread at once (window_mean then sums
+    // them in its fixed order from shared memory)
+    __shared__ double ring_s[3][DBW_DMAX];
+    for (int e = tid; e < 3 * DBW_DMAX; e += blockDim.x) {
+        const int r = e / DBW_DMAX, i = e - r * DBW_DMAX;
+        ring_s[r][i] = (r == 0 ? st->ringV : r == 1 ? st->ringN : st->ringL)[i];
+    }
+    __syncthreads();
     if (tid == 0) {
         int ready;
         const bool have_T = T_ext ? !isnan(T_ext[0]) : st->c > 0;
@@ -164,9 +182,9 @@ __global__ void __launch_bounds__(1024) choose_b_kernel(dbw_state* __restrict__ 
         } else {
             ready = st->cntV > 0 && st->cntN > 0 && st->cntL > 0 && st->c > 0 && have_T;
             if (ready) {
-                Vh_s = window_mean(st->ringV, st->cntV, st->D);   // Eq. (13)
-                Nh_s = window_mean(st->ringN, st->cntN, st->D);   // Eq. (14)
-                const double Lh = window_mean(st->ringL, st->cntL, st->D);   // Eq. (15)
+                Vh_s = window_mean(ring_s[0], st->cntV, st->D);   // Eq. (13)
+                Nh_s = window_mean(ring_s[1], st->cntN, st->D);   // Eq. (14)
+                const double Lh = window_mean(ring_s[2], st->cntL, st->D);   // Eq. (15)
                 q_s = ((Lh * lr) * lr) / 2.0;
             }
         }

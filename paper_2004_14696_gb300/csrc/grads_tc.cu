@@ -246,6 +246,8 @@ __global__ void __launch_bounds__(256) softmax_xent_ld_kernel(const float* __res
         worker = sel[i];
     }
     __shared__ int bad_s;
+    constexpr int kShared = 1024;   // sample losses kept in shared memory up to this B
+    __shared__ float ls[kShared];
     if (threadIdx.x == 0) bad_s = 0;
     __syncthreads();
     const float invB = 1.0f / static_cast<float>(B);
@@ -305,14 +307,17 @@ __global__ void __launch_bounds__(256) softmax_xent_ld_kernel(const float* __res
             }
         }
         if (lane == 0) {
-            sample_loss[row] = bad ? NAN : (mx + logf(se)) - z[y];
+            const float l = bad ? NAN : (mx + logf(se)) - z[y];
+            sample_loss[row] = l;
+            if (r < kShared) ls[r] = l;
             if (bad) bad_s = 1;
         }
     }
     __syncthreads();
     if (threadIdx.x == 0) {
+        // in sample order, from shared memory
         float acc = 0.f;
-        for (int r = 0; r < B; ++r) acc += sample_loss[static_cast<int64_t>(i) * B + r];
+        for (int r = 0; r < B; ++r) acc += r < kShared ? ls[r] : sample_loss[static_cast<int64_t>(i) * B + r];
         loss[worker] = bad_s ? NAN : acc * invB;
     }
     if (dZT) write_dzT(tileT, C, B, static_cast<int64_t>(i) * B, B, dZT, ldT);
@@ -470,8 +475,9 @@ struct FinishArgs {
 //   vals[n + 1] = ||g_t||^2 (all W and b pieces);
 //   vals[n] = sum_j ||g_j||^2 - k ||g_t||^2, the deviation sum of Eq. (10) by the
 //             identity sum_j ||g_j - g_t||^2 = sum_j ||g_j||^2 - k ||g_t||^2 (fp64).
-// Every sum runs in a fixed order (strided per thread, then a fixed tree).
-constexpr int kFinishThreads = 256;
+// Every sum runs in a fixed order (strided per thread, then a fixed tree).  1024
+// threads: the ~12k pieces of the 4096-wide workload are ~12 loads per thread.
+constexpr int kFinishThreads = 1024;
 
 __global__ void __launch_bounds__(kFinishThreads) finish_received_kernel(FinishArgs a, const int32_t* __restrict__ sel,
                                                                          const int* __restrict__ kdev,
