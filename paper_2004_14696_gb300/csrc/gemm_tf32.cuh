@@ -27,6 +27,22 @@
 namespace dbw {
 namespace tf32 {
 
+// Instruction descriptor of kind::tf32: D fp32 (bits 4-5 = 1), A and B tf32 (bits 7-9 = 2,
+// 10-12 = 2), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
+__host__ __device__ constexpr uint32_t instr_desc_tf32(int m, int n) {
+    return (1u << 4) | (2u << 7) | (2u << 10) | (static_cast<uint32_t>(n >> 3) << 17) |
+           (static_cast<uint32_t>(m >> 4) << 24);
+}
+// D (TMEM) (+)= A (tf32, shared memory) x B (tf32, shared memory): one K = 8 step.
+__device__ __forceinline__ void tc_mma_tf32(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
+        "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 constexpr int BM = 128;
 constexpr int kThreads = 192;
 constexpr int BK = 32;   // fp32 elements per 128-byte row
