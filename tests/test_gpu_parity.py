@@ -422,6 +422,42 @@ def test_worker_grads_parity_sampled_workers(wl):
                               workers, RTOL_BF16, gpu_active_sets(it.ws, wl.widths, wl.n, wl.B, wl.prec))
 
 
+def test_tf32_forward_on_eight_decades_of_magnitude():
+    """The fp32 forward GEMMs in three tf32 passes keep fp32 accuracy whatever the
+    operands' exponents: features of random sign and magnitude 10^U(-4, 4), every hidden
+    activation of layers 1 and 2 (both in three passes) within 1e-6 of the sum of
+    |terms| of its dot product, against the oracle's fp64 pre-activations (the level
+    measured on N(0,1) features is about 1e-7)."""
+    wl = TF32_RAGGED
+    it = Iteration(wl, static_b=0)
+    it.load_inputs(0)
+    rng = np.random.default_rng(4242)
+    S, F = it.pool.shape
+    pool = (rng.choice([-1.0, 1.0], size=(S, F)) * 10.0 ** rng.uniform(-4.0, 4.0, size=(S, F))).astype(np.float32)
+    it.pool.copy_(torch.from_numpy(pool))
+    dbw.dbw_worker_grads(wl.widths, wl.prec, it.w, it.pool, it.labels, it.idx, wl.n, wl.B, it.G, it.loss, it.ws)
+    torch.cuda.synchronize()
+    assert int(it.ws[:4].view(torch.int32).item()) == 0
+    acts = [dbw.hidden_activations(it.ws, wl.widths, wl.n, wl.B, wl.prec, h).cpu().numpy().astype(np.float64)
+            for h in (1, 2)]
+    idx, labels, w = it.idx.cpu().numpy(), it.labels.cpu().numpy(), it.w.cpu().numpy()
+    off1 = wl.widths[0] * wl.widths[1] + wl.widths[1]   # where layer 2's parameters start in w
+    worst = 0.0
+    for i in range(wl.n):
+        rows = slice(i * wl.B, (i + 1) * wl.B)
+        y = labels[idx[rows]]
+        # layer 1 from the features; layer 2 from the GPU's own layer-1 activations (the
+        # oracle's forward of the network above layer 1), so each GEMM is checked alone
+        _, _, z1, s1, _ = O.worker_grads(wl.widths, w, pool[idx[rows]].astype(np.float64), y, 1, wl.B, False,
+                                         return_preact=True, return_magnitude=True)
+        _, _, z2, s2, _ = O.worker_grads(wl.widths[1:], w[off1:], acts[0][rows], y, 1, wl.B, False,
+                                         return_preact=True, return_magnitude=True)
+        for z, sc, a in ((z1[0], s1[0], acts[0][rows]), (z2[0], s2[0], acts[1][rows])):
+            ratio = np.abs(np.maximum(z, 0.0) - a) / (1e-6 * sc)
+            worst = max(worst, float(ratio.max()))
+    assert worst <= 1.0, f"worst activation error {worst:.3g} x 1e-6 of its sum of |terms|"
+
+
 def test_bad_sample_index_poisons_only_that_worker():
     wl = SMALL_FP32_RAGGED
     it = Iteration(wl, static_b=0)
