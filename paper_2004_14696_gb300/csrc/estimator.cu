@@ -7,9 +7,11 @@
 // state reproduced elsewhere with the same operation order yields the same b_t
 // bit for bit.  The sequential pieces (window sums, the loss mean) run in one
 // thread on purpose: their summation order is part of that contract.  Their inputs
-// are first loaded into shared memory by all threads.
+// are first loaded into shared memory by all threads, and so are the state's scalar
+// fields (one round trip instead of one per field).
 #include <math.h>
 #include <math_constants.h>
+#include <stddef.h>
 
 #include "common.cuh"
 
@@ -26,6 +28,18 @@ __device__ double window_mean(const double* ring, int cnt, int D) {
     double acc = 0.0;
     for (int v = 1; v <= m; ++v) acc = acc + ring[ring_slot(cnt - v)];
     return acc / (double)m;
+}
+
+// The state's scalar fields (everything before the rings), copied into shared memory by
+// the first threads in one round trip; the sequential code then reads the copy and
+// writes its results to the state itself.
+constexpr int kHeadWords = static_cast<int>(offsetof(dbw_state, ringV) / 8);
+static_assert(offsetof(dbw_state, ringV) % 8 == 0, "the state's scalar fields are whole 8-byte words");
+
+__device__ __forceinline__ const dbw_state* stage_head(const dbw_state* st, unsigned long long* head) {
+    if (threadIdx.x < kHeadWords) head[threadIdx.x] = reinterpret_cast<const unsigned long long*>(st)[threadIdx.x];
+    __syncthreads();
+    return reinterpret_cast<const dbw_state*>(head);
 }
 
 // Sum of the per-block pieces of one quantity, in a fixed order: thread t adds
@@ -61,18 +75,19 @@ __global__ void __launch_bounds__(1024) grad_stats_kernel(
     // sequential sums from shared memory (n <= DBW_NMAX: checked by the caller)
     __shared__ uint8_t mask_s[DBW_NMAX];
     __shared__ float loss_s[DBW_NMAX];
+    __shared__ unsigned long long head_s[kHeadWords];
     const int tid = threadIdx.x;
     for (int j = tid; j < n; j += blockDim.x) {
         mask_s[j] = mask[j] ? 1 : 0;
         loss_s[j] = loss[j];
     }
-    __syncthreads();
+    const dbw_state* sh = stage_head(st, head_s);   // (its barrier also orders mask_s, loss_s)
     if (tid == 0) {
         int k = 0;
         for (int j = 0; j < n; ++j) k += mask_s[j];
         k_s = k;
-        if (k == 0 || st->n != n) {
-            st->flags |= (k == 0 ? DBW_FLAG_EMPTY_MASK : 0) | (st->n != n ? DBW_FLAG_BAD_STATE : 0);
+        if (k == 0 || sh->n != n) {
+            st->flags = sh->flags | (k == 0 ? DBW_FLAG_EMPTY_MASK : 0) | (sh->n != n ? DBW_FLAG_BAD_STATE : 0);
             k_s = 0;
         }
     }
@@ -95,23 +110,23 @@ __global__ void __launch_bounds__(1024) grad_stats_kernel(
         } else {
             flags |= DBW_FLAG_K1;
         }
-        if (st->t >= 1 && st->has_last) {                     // Eq. (12)
-            const double num = 2.0 * ((lr * st->N_last) - (st->F_last - F));
-            const double den = (lr * lr) * (st->N_last + (st->V_last / (double)st->k_last));
+        if (sh->t >= 1 && sh->has_last) {                     // Eq. (12)
+            const double num = 2.0 * ((lr * sh->N_last) - (sh->F_last - F));
+            const double den = (lr * lr) * (sh->N_last + (sh->V_last / (double)sh->k_last));
             if (den > 0.0) L = num / den;
             if (!(den > 0.0 && isfinite(L))) {
                 L = CUDART_NAN;
                 flags |= DBW_FLAG_L_SKIPPED;
             } else {
-                st->ringL[st->cntL % DBW_DMAX] = L;
-                st->cntL += 1;
+                st->ringL[sh->cntL % DBW_DMAX] = L;
+                st->cntL = sh->cntL + 1;
             }
         }
         if (k >= 2) {
-            st->ringV[st->cntV % DBW_DMAX] = V;
-            st->cntV += 1;
-            st->ringN[st->cntN % DBW_DMAX] = N;
-            st->cntN += 1;
+            st->ringV[sh->cntV % DBW_DMAX] = V;
+            st->cntV = sh->cntV + 1;
+            st->ringN[sh->cntN % DBW_DMAX] = N;
+            st->cntN = sh->cntN + 1;
             st->N_last = N;
             st->V_last = V;
             st->has_last = 1;
@@ -120,13 +135,14 @@ __global__ void __launch_bounds__(1024) grad_stats_kernel(
             st->V_last = CUDART_NAN;
             st->has_last = 0;
         }
-        st->c += 1;
-        st->vclock = st->vclock + tsorted[k - 1];
-        st->F_prev = st->F_last;
+        st->c = sh->c + 1;
+        const double vclock = sh->vclock + tsorted[k - 1];
+        st->vclock = vclock;
+        st->F_prev = sh->F_last;
         st->F_last = F;
         st->k_last = k;
-        st->t += 1;
-        st->flags |= flags;
+        st->t = sh->t + 1;
+        st->flags = sh->flags | flags;
         if (stats_out) {
             stats_out[DBW_STAT_K] = (double)k;
             stats_out[DBW_STAT_SS] = SS;
@@ -136,7 +152,7 @@ __global__ void __launch_bounds__(1024) grad_stats_kernel(
             stats_out[DBW_STAT_F] = F;
             stats_out[DBW_STAT_L] = L;
             stats_out[DBW_STAT_FLAGS] = (double)flags;
-            stats_out[DBW_STAT_VCLOCK] = st->vclock;
+            stats_out[DBW_STAT_VCLOCK] = vclock;
         }
     }
     // Sect. 3.2: every arrival is observed, S[r] accumulates the r-th order statistic
@@ -159,10 +175,12 @@ __global__ void __launch_bounds__(1024) choose_b_kernel(dbw_state* __restrict__ 
     __shared__ double best_r[32];
     __shared__ int best_k[32];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int n = st->n;
-    if (n < 1 || n > DBW_NMAX || st->D < 1 || st->D > DBW_DMAX || st->cntV < 0 || st->cntN < 0 ||
-        st->cntL < 0 || st->c < 0) {
-        if (tid == 0) st->flags |= DBW_FLAG_BAD_STATE;
+    __shared__ unsigned long long head_s[kHeadWords];
+    const dbw_state* sh = stage_head(st, head_s);
+    const int n = sh->n;
+    if (n < 1 || n > DBW_NMAX || sh->D < 1 || sh->D > DBW_DMAX || sh->cntV < 0 || sh->cntN < 0 ||
+        sh->cntL < 0 || sh->c < 0) {
+        if (tid == 0) st->flags = sh->flags | DBW_FLAG_BAD_STATE;
         return;
     }
     const bool blind = (flags & DBW_CHOOSE_BLIND) != 0;
@@ -176,15 +194,15 @@ __global__ void __launch_bounds__(1024) choose_b_kernel(dbw_state* __restrict__ 
     __syncthreads();
     if (tid == 0) {
         int ready;
-        const bool have_T = T_ext ? !isnan(T_ext[0]) : st->c > 0;
+        const bool have_T = T_ext ? !isnan(T_ext[0]) : sh->c > 0;
         if (blind) {
             ready = have_T;
         } else {
-            ready = st->cntV > 0 && st->cntN > 0 && st->cntL > 0 && st->c > 0 && have_T;
+            ready = sh->cntV > 0 && sh->cntN > 0 && sh->cntL > 0 && sh->c > 0 && have_T;
             if (ready) {
-                Vh_s = window_mean(ring_s[0], st->cntV, st->D);   // Eq. (13)
-                Nh_s = window_mean(ring_s[1], st->cntN, st->D);   // Eq. (14)
-                const double Lh = window_mean(ring_s[2], st->cntL, st->D);   // Eq. (15)
+                Vh_s = window_mean(ring_s[0], sh->cntV, sh->D);   // Eq. (13)
+                Nh_s = window_mean(ring_s[1], sh->cntN, sh->D);   // Eq. (14)
+                const double Lh = window_mean(ring_s[2], sh->cntL, sh->D);   // Eq. (15)
                 q_s = ((Lh * lr) * lr) / 2.0;
             }
         }
@@ -192,7 +210,7 @@ __global__ void __launch_bounds__(1024) choose_b_kernel(dbw_state* __restrict__ 
     }
     __syncthreads();
     const int ready = ready_s;
-    const double c = (double)st->c;
+    const double c = (double)sh->c;
     // candidate of this thread: k = tid + 1
     double my_r = -CUDART_INF;
     int my_k = 0;   // 0 = not eligible
@@ -242,8 +260,8 @@ __global__ void __launch_bounds__(1024) choose_b_kernel(dbw_state* __restrict__ 
             }
         }
         if (kstar == 0) kstar = n;                                // R3 / R7: k = n
-        if (st->t >= 2 && st->F_last > beta * st->F_prev && st->k_last < n) {   // Eq. (19)
-            const int kg = st->k_last + 1;
+        if (sh->t >= 2 && sh->F_last > beta * sh->F_prev && sh->k_last < n) {   // Eq. (19)
+            const int kg = sh->k_last + 1;
             if (kg > kstar) kstar = kg;
         }
         if (kstar > n) kstar = n;

@@ -570,6 +570,49 @@ __global__ void __launch_bounds__(256) skinny_n_kernel(int M, int N, int K, cons
     }
 }
 
+// The same for fp32 operands whose rows allow 16-byte loads (K, lda, ldw multiples of 4,
+// A and W 16-byte aligned): no shared memory, W read through L1; lane l takes the
+// 4-element groups k = 4 l, 4 l + 128, .. of its row, each group's products added in k
+// order, then the butterfly.
+template <class Epi>
+__global__ void __launch_bounds__(128) skinny_n4_kernel(int M, int N, int K, const float* __restrict__ A, int64_t lda,
+                                                        const float* __restrict__ W, int64_t ldw, Epi epi) {
+    const int lane = threadIdx.x & 31;
+    const int nwarps = (gridDim.x * blockDim.x) >> 5;
+    for (int m = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; m < M; m += nwarps) {
+        float acc[kSkinnyN];
+#pragma unroll
+        for (int n = 0; n < kSkinnyN; ++n) acc[n] = 0.f;
+        const float* a = A + (int64_t)m * lda;
+        for (int k = 4 * lane; k < K; k += 128) {
+            const float4 av = __ldg(reinterpret_cast<const float4*>(a + k));
+#pragma unroll
+            for (int n = 0; n < kSkinnyN; ++n) {
+                if (n < N) {
+                    const float4 wv = __ldg(reinterpret_cast<const float4*>(W + (int64_t)n * ldw + k));
+                    float t = acc[n];
+                    t = fmaf(av.x, wv.x, t);
+                    t = fmaf(av.y, wv.y, t);
+                    t = fmaf(av.z, wv.z, t);
+                    t = fmaf(av.w, wv.w, t);
+                    acc[n] = t;
+                }
+            }
+        }
+        float mine = 0.f;
+#pragma unroll
+        for (int n = 0; n < kSkinnyN; ++n) {
+            if (n < N) {
+                float v = acc[n];
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+                if (lane == n) mine = v;
+            }
+        }
+        if (lane < N) epi(0, m, lane, mine);
+    }
+}
+
 // Input-gradient GEMM with a short inner dimension (K = out <= kSkinnyK):
 // dZ_{l-1}[m, c] = (sum_{o < K} dZ_l[m, o] W[o, c]) * 1[act[m, c] > 0], the products
 // added in increasing o (EpiDx's arithmetic, with the 16 masks loaded before any
@@ -697,6 +740,15 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
                 if (tc)
                     return tf32::run(M, fout, fin, Ain, fin, W, fin, part[0], part[1], part[2], part[3], epi, status,
                                      st, /*a_parts_ready=*/l == 0);
+            }
+            if constexpr (sizeof(T) == 4) {
+                if (fout <= kSkinnyN && fin % 4 == 0 && aligned16(Ain) && aligned16(W)) {
+                    const int want = (M + 3) / 4;   // 4 rows (warps) per CTA
+                    const int grid = want < 8 * sm_count() ? want : 8 * sm_count();
+                    skinny_n4_kernel<<<grid, 128, 0, st>>>(M, fout, fin, reinterpret_cast<const float*>(Ain), fin,
+                                                           reinterpret_cast<const float*>(W), fin, epi);
+                    return cudaGetLastError();
+                }
             }
             if (skinny_n_ok(fout, fin)) {
                 const int rows_per_cta = 8;

@@ -228,8 +228,9 @@ class Iteration:
             kps = -(-(-(-k // s)) // 16) * 16
             return 1 if -(-k // kps) > 1 else 0
 
-        def skinny_n(n, k):     # the forward GEMM with few outputs
-            return n <= 16 and n * k * 4 <= 48 * 1024
+        def skinny_n(n, k, off):     # the forward GEMM with few outputs (W_l at offset off of w)
+            vec = self.wl.prec == dbw.PREC_FP32 and k % 4 == 0 and off % 4 == 0
+            return n <= 16 and (vec or n * k * 4 <= 48 * 1024)
 
         def skinny_k(n, k):     # the input-gradient GEMM with a short inner dimension
             return k <= 32 and (n + 16) * k * 4 <= 48 * 1024
@@ -241,11 +242,11 @@ class Iteration:
             if (self.wl.prec == dbw.PREC_FP32 and B % 32 == 0 and B <= 256 and fin % 4 == 0 and off % 4 == 0
                     and fout >= 32 and n * fout * fin * B >= 1 << 25):
                 extra += 1 if l == 0 else 2     # transposed parts of dZ_l (and of the input above layer 1)
-            off += fin * fout + fout
             if self.wl.prec == dbw.PREC_FP32 and fout >= 32 and M * fout * fin >= 1 << 27:
                 extra += 1 if l == 0 else 2     # the gather writes the first layer's input parts
-            elif not skinny_n(fout, fin):
+            elif not skinny_n(fout, fin, off):
                 extra += split_launch(M, fout, fin)
+            off += fin * fout + fout
             if l > 0 and not skinny_k(fin, fout):
                 extra += split_launch(M, fin, fout)
         return extra
