@@ -153,7 +153,12 @@ size_t dbw_worker_grads_workspace_bytes(int num_layers, const int32_t* widths, i
  *          success, bit 0 set if a tensor-core pipeline wait timed out (it is
  *          bounded, never a hang), in which case G and loss are undefined.
  *  Path: with prec = DBW_PREC_BF16 and B a multiple of 32 the GEMMs run on
- *  the tcgen05 tensor cores; otherwise on fp32 FFMA (SIMT) tiles.
+ *  the tcgen05 tensor cores in bf16.  With prec = DBW_PREC_FP32 the large
+ *  forward and per-worker weight-gradient GEMMs run on the tcgen05 tensor
+ *  cores in three tf32 passes (fp32 accuracy: each operand split into two
+ *  tf32 parts), small-output and short-inner-dimension GEMMs on dedicated
+ *  kernels, the rest on fp32 FFMA (SIMT) tiles; bf16 with B % 32 != 0 runs
+ *  on the SIMT tiles too.
  *  prec    DBW_PREC_FP32 or DBW_PREC_BF16.
  */
 int dbw_worker_grads(int num_layers, const int32_t* widths, int prec,
