@@ -365,6 +365,10 @@ WIDE_BF16 = workloads.Workload(
     key="wide_bf16", widths=(64, 320), n=2, B=256, prec=workloads.PREC_BF16, S=600,
     feature_dist="normal", time_model="shifted_exp", time_params={"shift": 1.0, "rate": 1.0}, lr=0.01,
     seed_offset=82)
+# one layer, 7 classes, 132 features: the 16-byte logits kernel on a ragged one-layer shape
+SMALL_FP32_LINEAR = workloads.Workload(
+    key="small_fp32_linear", widths=(132, 7), n=5, B=3, prec=workloads.PREC_FP32, S=50,
+    feature_dist="uniform", time_model="pareto", time_params={"alpha": 2.0, "xm": 1.0}, lr=0.05, seed_offset=85)
 SMALL_FP32_RAGGED = workloads.Workload(
     key="small_fp32", widths=(132, 200, 70, 7), n=5, B=3, prec=workloads.PREC_FP32, S=50,
     feature_dist="uniform", time_model="pareto", time_params={"alpha": 2.0, "xm": 1.0}, lr=0.05, seed_offset=78)
@@ -396,8 +400,9 @@ def grads_case(wl, t=0):
     return it, idx
 
 
-@pytest.mark.parametrize("wl", [workloads.SOFTMAX784, workloads.MLP784, SMALL_FP32_RAGGED, TF32_RAGGED, TF32_DW,
-                                SMALL_BF16, SMALL_BF16_SIMT, ODD_BF16, UNALIGNED_BF16, WIDE_BF16],
+@pytest.mark.parametrize("wl", [workloads.SOFTMAX784, SMALL_FP32_LINEAR, workloads.MLP784, SMALL_FP32_RAGGED,
+                                TF32_RAGGED, TF32_DW, SMALL_BF16, SMALL_BF16_SIMT, ODD_BF16, UNALIGNED_BF16,
+                                WIDE_BF16],
                          ids=lambda w: w.key)
 def test_worker_grads_parity_full(wl):
     it, idx = grads_case(wl)
@@ -458,8 +463,8 @@ def test_tf32_forward_on_eight_decades_of_magnitude():
     assert worst <= 1.0, f"worst activation error {worst:.3g} x 1e-6 of its sum of |terms|"
 
 
-def test_bad_sample_index_poisons_only_that_worker():
-    wl = SMALL_FP32_RAGGED
+@pytest.mark.parametrize("wl", [SMALL_FP32_RAGGED, SMALL_FP32_LINEAR], ids=lambda w: w.key)
+def test_bad_sample_index_poisons_only_that_worker(wl):
     it = Iteration(wl, static_b=0)
     idx, _ = it.host_inputs(0)
     idx[wl.B + 1] = wl.S + 7          # worker 1 gets an out-of-range sample
