@@ -1,5 +1,6 @@
-// fp32 GEMM on the tcgen05 tensor cores in three tf32 passes (3xTF32), for the fp32
-// workloads' forward GEMMs.  Internal header (templates on the epilogue).
+// fp32 GEMMs on the tcgen05 tensor cores in three tf32 passes (3xTF32), for the fp32
+// workloads: the forward GEMM (gemm_kernel, templated on its epilogue) and the per-worker
+// weight gradient written into G (dw_kernel).  Internal header, included by grads.cu only.
 //
 // Every fp32 operand x is split into hi = x rounded to nearest tf32 (10 mantissa bits)
 // and lo = x - hi (exact in fp32, |lo| <= 2^-11 |x|), itself stored rounded to nearest
@@ -14,7 +15,7 @@
 // and the epilogue adds the NMAIN + 1 partial sums in fp32, rounding to nearest.  Each
 // accumulator then takes about K / (8 NMAIN) MMA additions instead of 3 K / 8.
 //
-// One CTA per 128 x BN output tile (the single-CTA layout of tc_gemm_kernel): a TMA
+// gemm_kernel: one CTA per 128 x BN output tile (the single-CTA layout of tc_gemm_kernel): a TMA
 // producer thread, an MMA thread, four epilogue warps (one per 32-row TMEM lane
 // quarter).  A stage holds 32-deep K slices of A_hi, A_lo (128 rows) and B_hi, B_lo
 // (BN rows), 128-byte swizzled; its 4 K = 8 steps issue 3 MMAs each.  Every wait is
