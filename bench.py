@@ -83,6 +83,7 @@ def parse():
     # single pieces
     p.add_argument("--case", choices=CASES)
     p.add_argument("--n", type=int, default=64)
+    p.add_argument("--tol", type=float, default=1e-4, help="--case psw: stopping tolerance of the Eq. (17) fit")
     p.add_argument("--d", type=int, default=4_000_000)
     p.add_argument("--b", type=int, default=16)
     p.add_argument("--reps", type=int, default=5)
@@ -646,7 +647,7 @@ def received_case(key, b, reps):
     return out
 
 
-def psw_case(n, iters, seed=2004146971, model="pareto", tol=1e-6):
+def psw_case(n, iters, seed=2004146971, model="pareto", tol=1e-4):
     """The push-and-wait clock and the Eq. (17) fit alone, per iteration: arrivals,
     selection, record and the warm-started fit, with k_t drawn uniformly from 1..n
     (every row of the cell table gets samples, the hardest case for the fit)."""
@@ -890,7 +891,7 @@ def run_case(args):
     elif args.case == "received":
         print(json.dumps(received_case(args.workload, args.b, args.reps)), flush=True)
     elif args.case == "psw":
-        print(json.dumps(psw_case(args.n, args.iters)), flush=True)
+        print(json.dumps(psw_case(args.n, args.iters, tol=args.tol)), flush=True)
     else:
         print(json.dumps(iterate_case(args.workload, args.iters, args.warmup, args.received, args.graph)), flush=True)
 

@@ -26,7 +26,7 @@ from .workloads import Workload
 
 class Iteration:
     def __init__(self, wl: Workload, device="cuda", static_b=None, blind=False, keep_gbar=False,
-                 pool=None, labels=None, w0=None, received=False, clock="psi", psw_tol=1e-6,
+                 pool=None, labels=None, w0=None, received=False, clock="psi", psw_tol=1e-4,
                  psw_max_sweeps=100000):
         self.wl = wl
         self.device = torch.device(device)

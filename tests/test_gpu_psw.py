@@ -121,18 +121,20 @@ def assert_fit_close(got, ref, what):
     assert np.all(err <= lim), (what, float(np.max(err / np.where(lim > 0, lim, np.inf))))
 
 
+@pytest.mark.parametrize("tol", [1e-6, 1e-4])
 @pytest.mark.parametrize("n,steps", [(16, 40), (64, 30), (256, 12)])
-def test_time_estimates_match_the_oracle(n, steps):
+def test_time_estimates_match_the_oracle(n, steps, tol):
     """T^_k after several iterations (the GPU fit is warm-started from the previous
     one, the oracle's is not) against the oracle's, element by element within 1e-5 of
     each value.  The fp32 sweeps find the blocks of the solution; their values are
-    the exact fp64 means of the blocks' samples."""
+    the exact fp64 means of the blocks' samples.  So a looser stopping tolerance
+    (1e-4, the pipeline's) gives the same values once the sweeps have found the blocks."""
     c = Clock(n)
     ks = k_sequence(n, steps, 3)
     T = torch.empty(n, dtype=torch.float64, device="cuda")
     for t in range(steps):
         c.step(inputs.completion_times(11, t, n, "pareto", alpha=2.0, xm=1.0), ks[t])
-        dbw.dbw_psw_estimate(c.psw, n, T, tol=1e-6, max_sweeps=200000)
+        dbw.dbw_psw_estimate(c.psw, n, T, tol=tol, max_sweeps=200000)
         if t in (0, 1, 4, steps // 2, steps - 1):
             torch.cuda.synchronize()
             ref = np.array(P.time_estimates(c.ps))
@@ -272,8 +274,9 @@ def psw_margin(st, lr, beta, T):
     return min(gaps)
 
 
+@pytest.mark.parametrize("tol", [1e-6, 1e-4])
 @pytest.mark.parametrize("n", [96, 200])
-def test_fit_on_planted_tables(n):
+def test_fit_on_planted_tables(n, tol):
     """Eq. (17) on cell tables written straight into the state, shaped so that the split
     chains pool across their parts: group rows whose cell means fall along the whole row
     (one block absorbs every part), rise (nothing pools), or zig-zag, with random counts;
@@ -311,7 +314,7 @@ def test_fit_on_planted_tables(n):
     ps.sums[1:, 1:] = sums.astype(np.float64) * unit
     ps.cnts[1:, 1:] = cnts
     T = torch.empty(n, dtype=torch.float64, device="cuda")
-    dbw.dbw_psw_estimate(psw, n, T, tol=1e-6, max_sweeps=200000)
+    dbw.dbw_psw_estimate(psw, n, T, tol=tol, max_sweeps=200000)
     torch.cuda.synchronize()
     g = dbw.read_psw(psw, n)
     assert not (g["flags"] & (dbw.PSW_NOT_CONVERGED | dbw.PSW_UNPOLISHED)), g["flags"]
