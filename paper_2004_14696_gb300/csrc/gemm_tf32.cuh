@@ -273,19 +273,26 @@ cudaError_t run(int M, int N, int K, const float* A, int64_t lda, const float* B
 // the in-tiles fastest; each tile has a hi.hi accumulator and a correction accumulator
 // (256 TMEM columns), two tiles in flight (512 columns), so that the MMAs of tile i + 1
 // run while the epilogue drains tile i.  With K = B <= 256 the hi.hi accumulator takes at
-// most 32 MMA additions.  Four epilogue warps, one per TMEM lane quarter (32 G rows),
-// each copy their 32 x 128 block TMEM -> registers (hi.hi + corrections, rounded to
-// nearest) -> shared memory (16-byte pieces XOR-swizzled by row) and then store it row by
-// row, 512 contiguous bytes of one G row per instruction.
+// most 32 MMA additions.  Eight epilogue warps, two per TMEM lane quarter (32 G rows),
+// each copy their 32 x 64 block TMEM -> registers (hi.hi + corrections, rounded to
+// nearest; its four TMEM loads in flight together) -> shared memory (16-byte pieces
+// XOR-swizzled by row) and then store it, 256 contiguous bytes of each of two G rows per
+// instruction.
 namespace dw {
 constexpr int BN = 128;
 constexpr int STAGES = 2;
-constexpr int EPI_WARPS = 4;
+constexpr int EPI_WARPS = 8;                             // two per TMEM lane quarter (16 measured slower)
 constexpr int THREADS = 32 * (2 + EPI_WARPS);
 constexpr int A_BYTES = BM * BK * 4;
 constexpr int B_BYTES = BN * BK * 4;
 constexpr int STAGE_BYTES = 2 * A_BYTES + 2 * B_BYTES;   // A_hi, A_lo, B_hi, B_lo
-constexpr int WARP_STAGING = 32 * BN * 4;                // 32 rows x 512 bytes
+constexpr int WARP_COLS = BN / (EPI_WARPS / 4);          // columns of the tile per epilogue warp
+constexpr int NSEG = WARP_COLS / 32;                     // its 32-column TMEM segments
+constexpr int ROW_BYTES = WARP_COLS * 4;                 // a staged row
+constexpr int LANES_PER_ROW = WARP_COLS / 4;             // 16-byte pieces of a row
+constexpr int ROWS_PER_STORE = 32 / LANES_PER_ROW;       // rows one store instruction covers
+constexpr int WARP_STAGING = 32 * ROW_BYTES;
+static_assert(WARP_COLS % 32 == 0 && EPI_WARPS % 4 == 0, "whole 32-column segments per epilogue warp");
 constexpr int SMEM = STAGES * STAGE_BYTES + EPI_WARPS * WARP_STAGING + 256 + 1024;
 constexpr int TILE_COLS = 2 * BN;                         // hi.hi, then the corrections
 constexpr int TMEM_COLS = 2 * TILE_COLS;
@@ -411,7 +418,8 @@ static __global__ void __launch_bounds__(dw::THREADS, 1)
         }
     } else if (warp >= 2) {
         // ---------------- epilogue
-        const int q = warp & 3;   // TMEM lanes 32 q .. 32 q + 31 = G rows m0 + 32 q ..
+        const int q = warp & 3;          // TMEM lanes 32 q .. 32 q + 31 = G rows m0 + 32 q ..
+        const int h = (warp - 2) >> 2;   // columns [WARP_COLS h, WARP_COLS (h + 1)) of the tile
         uint8_t* buf = staging + (warp - 2) * dw::WARP_STAGING;
         int i = 0;
         for (long long t = blockIdx.x; t < total; t += gridDim.x, ++i) {
@@ -430,37 +438,45 @@ static __global__ void __launch_bounds__(dw::THREADS, 1)
             const uint32_t tbase =
                 tmem + static_cast<uint32_t>(acc * dw::TILE_COLS) + (static_cast<uint32_t>(q * 32) << 16);
             const int row0 = m0 + q * 32;
-            if (row0 < Mr) {
-                // TMEM -> smem: lane = row; piece p of 128-byte segment sgm of row r at
-                // r * 512 + sgm * 128 + ((p ^ (r & 7)) * 16)
-#pragma unroll 1
-                for (int sgm = 0; sgm < dw::BN / 32; ++sgm) {
-                    uint32_t rm[32], rc[32];
-                    tc_ld_32cols(tbase + sgm * 32, rm);
-                    tc_ld_32cols(tbase + dw::BN + sgm * 32, rc);
-                    tc_wait_ld();
+            const int c0 = h * dw::WARP_COLS;   // this warp's first column of the tile
+            if (row0 < Mr && n0 + c0 < Nr) {
+                // TMEM -> smem, every segment's loads in flight together: lane = row; piece p of
+                // 128-byte segment s of row r at r * ROW_BYTES + s * 128 + ((p ^ (r & 7)) * 16)
+                uint32_t rm[dw::NSEG][32], rc[dw::NSEG][32];
+#pragma unroll
+                for (int sg = 0; sg < dw::NSEG; ++sg) {
+                    tc_ld_32cols(tbase + c0 + 32 * sg, rm[sg]);
+                    tc_ld_32cols(tbase + dw::BN + c0 + 32 * sg, rc[sg]);
+                }
+                tc_wait_ld();
+#pragma unroll
+                for (int sg = 0; sg < dw::NSEG; ++sg) {
 #pragma unroll
                     for (int pc = 0; pc < 8; ++pc) {
                         float4 v;
-                        v.x = u2f(rm[4 * pc]) + u2f(rc[4 * pc]);
-                        v.y = u2f(rm[4 * pc + 1]) + u2f(rc[4 * pc + 1]);
-                        v.z = u2f(rm[4 * pc + 2]) + u2f(rc[4 * pc + 2]);
-                        v.w = u2f(rm[4 * pc + 3]) + u2f(rc[4 * pc + 3]);
-                        *reinterpret_cast<float4*>(buf + lane * 512 + sgm * 128 + ((pc ^ (lane & 7)) << 4)) = v;
+                        v.x = u2f(rm[sg][4 * pc]) + u2f(rc[sg][4 * pc]);
+                        v.y = u2f(rm[sg][4 * pc + 1]) + u2f(rc[sg][4 * pc + 1]);
+                        v.z = u2f(rm[sg][4 * pc + 2]) + u2f(rc[sg][4 * pc + 2]);
+                        v.w = u2f(rm[sg][4 * pc + 3]) + u2f(rc[sg][4 * pc + 3]);
+                        *reinterpret_cast<float4*>(buf + lane * dw::ROW_BYTES + sg * 128 + ((pc ^ (lane & 7)) << 4)) =
+                            v;
                     }
                 }
                 __syncwarp();
-                // smem -> G, one row per instruction: lane L writes columns n0 + 4 L .. + 3
-                const int sgm = lane >> 3, pc = lane & 7;
-                const int col = n0 + 4 * lane;
+                // smem -> G, ROWS_PER_STORE rows per instruction: a lane writes columns
+                // n0 + c0 + 4 piece .. + 3 of row rr + ro (ROW_BYTES contiguous bytes of each row)
+                const int ro = lane / dw::LANES_PER_ROW, piece = lane % dw::LANES_PER_ROW;
+                const int sg = piece >> 3, pc = piece & 7;
+                const int col = n0 + c0 + 4 * piece;
                 const bool col_ok = col + 3 < Nr;   // Nr % 4 == 0: whole pieces in or out
                 float* gcol = Gbase + static_cast<int64_t>(z) * ldG + col;
 #pragma unroll 4
-                for (int rr = 0; rr < 32; ++rr) {
+                for (int rr = 0; rr < 32; rr += dw::ROWS_PER_STORE) {
+                    const int r = rr + ro;
                     const float4 v =
-                        *reinterpret_cast<const float4*>(buf + rr * 512 + sgm * 128 + ((pc ^ (rr & 7)) << 4));
-                    if (col_ok && row0 + rr < Mr)
-                        __stcs(reinterpret_cast<float4*>(gcol + static_cast<int64_t>(row0 + rr) * ldrow), v);
+                        *reinterpret_cast<const float4*>(buf + r * dw::ROW_BYTES + sg * 128 + ((pc ^ (r & 7)) << 4));
+                    if (col_ok && row0 + r < Mr)
+                        __stcs(reinterpret_cast<float4*>(gcol + static_cast<int64_t>(row0 + r) * ldrow), v);
                 }
                 __syncwarp();
             }
