@@ -143,35 +143,49 @@ __global__ void gather_kernel(const float* __restrict__ pool, int64_t S, int in,
 
 // The gather of the fp32 pass when its first layer runs in three tf32 passes: the
 // gathered rows' tf32 parts row-major (hi / lo [M, ldo], when hi != nullptr) and
-// transposed (hiT / loT [in, ldt], when hiT != nullptr), and X itself when X != nullptr;
-// 32 x 32 tiles of X through shared memory, blocks of 32 x 8 threads.
+// transposed (hiT / loT [in, ldt], when hiT != nullptr), and X itself when X != nullptr.
+// Tiles of 32 rows x 128 columns through shared memory, blocks of 32 x 8 threads: a lane
+// moves 16 bytes of a row (in, ldo multiples of 4), then 4-byte pieces of the transposed
+// rows, 128 contiguous bytes a warp.
 __global__ void gather_parts_kernel(const float* __restrict__ pool, int64_t S, int in,
                                     const int32_t* __restrict__ idx, int M, float* __restrict__ X,
                                     float* __restrict__ hi, float* __restrict__ lo, int64_t ldo,
                                     float* __restrict__ hiT, float* __restrict__ loT, int64_t ldt) {
-    __shared__ float tile[32][33];
+    __shared__ float tile[32][129];   // [row][column], padded: the transposed reads are conflict-free
     const int tx = threadIdx.x, ty = threadIdx.y;
-    const int c0 = blockIdx.x * 32;
+    const int c0 = blockIdx.x * 128;
     for (int64_t m0 = (int64_t)blockIdx.y * 32; m0 < M; m0 += (int64_t)gridDim.y * 32) {
         for (int j = ty; j < 32; j += 8) {
             const int64_t m = m0 + j;
-            const int c = c0 + tx;
-            float v = 0.f;
+            const int c = c0 + 4 * tx;
+            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
             if (m < M && c < in) {
                 int64_t r = idx[m];
                 if (r < 0 || r >= S) r = 0;
-                v = pool[r * in + c];
-                if (X) X[m * in + c] = v;
-                if (hi) tf32::split_value(v, hi[m * ldo + c], lo[m * ldo + c]);
+                v = *reinterpret_cast<const float4*>(pool + r * in + c);
+                if (X) *reinterpret_cast<float4*>(X + m * in + c) = v;
+                if (hi) {
+                    float4 h, l;
+                    tf32::split_value(v.x, h.x, l.x);
+                    tf32::split_value(v.y, h.y, l.y);
+                    tf32::split_value(v.z, h.z, l.z);
+                    tf32::split_value(v.w, h.w, l.w);
+                    *reinterpret_cast<float4*>(hi + m * ldo + c) = h;
+                    *reinterpret_cast<float4*>(lo + m * ldo + c) = l;
+                }
             }
-            tile[j][tx] = v;
+            tile[j][4 * tx] = v.x;
+            tile[j][4 * tx + 1] = v.y;
+            tile[j][4 * tx + 2] = v.z;
+            tile[j][4 * tx + 3] = v.w;
         }
         if (hiT) {
             __syncthreads();
-            for (int j = ty; j < 32; j += 8) {
-                const int c = c0 + j;
+            for (int cc = ty; cc < 128; cc += 8) {
+                const int c = c0 + cc;
                 const int64_t m = m0 + tx;
-                if (c < in && m < M) tf32::split_value(tile[tx][j], hiT[(int64_t)c * ldt + m], loT[(int64_t)c * ldt + m]);
+                if (c < in && m < M)
+                    tf32::split_value(tile[tx][cc], hiT[(int64_t)c * ldt + m], loT[(int64_t)c * ldt + m]);
             }
             __syncthreads();
         }
@@ -707,7 +721,7 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
             // X itself only when one of them stays on SIMT
             const int ty = (M + 31) / 32;
             const bool need_x = !(P.tf32[0] && P.tf32_dw[0]);
-            gather_parts_kernel<<<dim3((in + 31) / 32, ty < 65535 ? ty : 65535), dim3(32, 8), 0, st>>>(
+            gather_parts_kernel<<<dim3((in + 127) / 128, ty < 65535 ? ty : 65535), dim3(32, 8), 0, st>>>(
                 pool, S, in, idx, M, need_x ? reinterpret_cast<float*>(X) : nullptr,
                 P.tf32[0] ? reinterpret_cast<float*>(ws + P.off_ahi) : nullptr,
                 P.tf32[0] ? reinterpret_cast<float*>(ws + P.off_alo) : nullptr, (in + 3) / 4 * 4,
