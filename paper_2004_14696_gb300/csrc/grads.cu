@@ -588,7 +588,9 @@ __global__ void __launch_bounds__(256) skinny_n_kernel(int M, int N, int K, cons
 // A and W 16-byte aligned): no shared memory, W read through L1; lane l takes the
 // 4-element groups k = 4 l, 4 l + 128, .. of its row, each group's products added in k
 // order, then the butterfly.
-template <class Epi>
+// kTwo: two groups per pass with all their loads issued first (fewer round trips for long
+// rows, at about 160 registers); else one group per pass (few registers, for K <= 256).
+template <bool kTwo, class Epi>
 __global__ void __launch_bounds__(128) skinny_n4_kernel(int M, int N, int K, const float* __restrict__ A, int64_t lda,
                                                         const float* __restrict__ W, int64_t ldw, Epi epi) {
     const int lane = threadIdx.x & 31;
@@ -598,18 +600,54 @@ __global__ void __launch_bounds__(128) skinny_n4_kernel(int M, int N, int K, con
 #pragma unroll
         for (int n = 0; n < kSkinnyN; ++n) acc[n] = 0.f;
         const float* a = A + (int64_t)m * lda;
-        for (int k = 4 * lane; k < K; k += 128) {
-            const float4 av = __ldg(reinterpret_cast<const float4*>(a + k));
+        if constexpr (kTwo) {
+            // two of the lane's 4-element groups per pass, all their loads issued before the
+            // products (which are added in group order, as below)
+            for (int k0 = 4 * lane; k0 < K; k0 += 256) {
+                const bool two = k0 + 128 < K;
+                const float4 av0 = __ldg(reinterpret_cast<const float4*>(a + k0));
+                const float4 av1 =
+                    two ? __ldg(reinterpret_cast<const float4*>(a + k0 + 128)) : make_float4(0.f, 0.f, 0.f, 0.f);
+                float4 wv0[kSkinnyN], wv1[kSkinnyN];
 #pragma unroll
-            for (int n = 0; n < kSkinnyN; ++n) {
-                if (n < N) {
-                    const float4 wv = __ldg(reinterpret_cast<const float4*>(W + (int64_t)n * ldw + k));
-                    float t = acc[n];
-                    t = fmaf(av.x, wv.x, t);
-                    t = fmaf(av.y, wv.y, t);
-                    t = fmaf(av.z, wv.z, t);
-                    t = fmaf(av.w, wv.w, t);
-                    acc[n] = t;
+                for (int n = 0; n < kSkinnyN; ++n) {
+                    if (n < N) {
+                        wv0[n] = __ldg(reinterpret_cast<const float4*>(W + (int64_t)n * ldw + k0));
+                        if (two) wv1[n] = __ldg(reinterpret_cast<const float4*>(W + (int64_t)n * ldw + k0 + 128));
+                    }
+                }
+#pragma unroll
+                for (int n = 0; n < kSkinnyN; ++n) {
+                    if (n < N) {
+                        float t = acc[n];
+                        t = fmaf(av0.x, wv0[n].x, t);
+                        t = fmaf(av0.y, wv0[n].y, t);
+                        t = fmaf(av0.z, wv0[n].z, t);
+                        t = fmaf(av0.w, wv0[n].w, t);
+                        if (two) {
+                            t = fmaf(av1.x, wv1[n].x, t);
+                            t = fmaf(av1.y, wv1[n].y, t);
+                            t = fmaf(av1.z, wv1[n].z, t);
+                            t = fmaf(av1.w, wv1[n].w, t);
+                        }
+                        acc[n] = t;
+                    }
+                }
+            }
+        } else {
+            for (int k = 4 * lane; k < K; k += 128) {
+                const float4 av = __ldg(reinterpret_cast<const float4*>(a + k));
+#pragma unroll
+                for (int n = 0; n < kSkinnyN; ++n) {
+                    if (n < N) {
+                        const float4 wv = __ldg(reinterpret_cast<const float4*>(W + (int64_t)n * ldw + k));
+                        float t = acc[n];
+                        t = fmaf(av.x, wv.x, t);
+                        t = fmaf(av.y, wv.y, t);
+                        t = fmaf(av.z, wv.z, t);
+                        t = fmaf(av.w, wv.w, t);
+                        acc[n] = t;
+                    }
                 }
             }
         }
@@ -759,8 +797,12 @@ int worker_grads_impl(const GradsPlan& P, const float* w, const float* pool, int
                 if (fout <= kSkinnyN && fin % 4 == 0 && aligned16(Ain) && aligned16(W)) {
                     const int want = (M + 3) / 4;   // 4 rows (warps) per CTA
                     const int grid = want < 8 * sm_count() ? want : 8 * sm_count();
-                    skinny_n4_kernel<<<grid, 128, 0, st>>>(M, fout, fin, reinterpret_cast<const float*>(Ain), fin,
-                                                           reinterpret_cast<const float*>(W), fin, epi);
+                    if (fin > 256)
+                        skinny_n4_kernel<true><<<grid, 128, 0, st>>>(M, fout, fin, reinterpret_cast<const float*>(Ain),
+                                                                     fin, reinterpret_cast<const float*>(W), fin, epi);
+                    else
+                        skinny_n4_kernel<false><<<grid, 128, 0, st>>>(M, fout, fin, reinterpret_cast<const float*>(Ain),
+                                                                      fin, reinterpret_cast<const float*>(W), fin, epi);
                     return cudaGetLastError();
                 }
             }
